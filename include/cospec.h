@@ -1,0 +1,214 @@
+/*
+ * cospec.h -- C ABI of the GB300 (sm_103a) verify/arbitrate round of
+ * collaborative speculative decoding (CoSpec).
+ *
+ * One round (Sec. 3.1 and Sec. 3.3 of the paper; App. F, Inference Procedure):
+ *   1. cospec_verify_attn            per layer: attention of the K+1 block rows
+ *                                    over a paged bf16 KV cache (Eq. 2)
+ *   2. cospec_lmhead_argmax_features LM head fused with argmax and the
+ *                                    log-prob statistics (Eq. 2, Eq. 23)
+ *   3. cospec_arbitrate              accept/reject at every draft/target
+ *                                    mismatch (Eq. 3, Eq. 13-14, Eq. 17)
+ *   4. cospec_accept_commit          accepted length and emitted tokens
+ *                                    (Eq. 15), KV commit of the accepted rows
+ *
+ * Conventions shared by every call
+ *  - Every array pointer is a DEVICE pointer owned by the caller; the library
+ *    allocates nothing, frees nothing and never synchronises the stream,
+ *    except cospec_get_device_error.  `stream` is a cudaStream_t (NULL = the
+ *    legacy default stream).  All calls are asynchronous.
+ *  - bf16 tensors are passed as uint16_t bit patterns, row-major, innermost
+ *    dimension last, densely packed.
+ *  - Host-side argument checks run before anything is launched; a failing
+ *    check returns a negative cospec_status and launches nothing.
+ *  - Data-dependent violations found on the device (a page id outside the
+ *    pool, a context that does not fit its page-table row, a token id outside
+ *    the vocabulary, a pipeline wait that timed out) skip the offending unit
+ *    and set a bit in a device error word (COSPEC_DEVERR_*), which
+ *    cospec_get_device_error reads and clears.  No kernel traps.
+ *  - Block geometry: a round verifies R = K + 1 rows per sequence.  Row 0 is
+ *    the last token emitted by the previous round (its KV is not committed
+ *    yet), rows 1..K are the draft tokens y_hat_1..y_hat_K.  Row j sits at
+ *    absolute position ctx_len[b] + j and its LM-head row predicts
+ *    y_tilde_{j+1}.
+ */
+#ifndef COSPEC_H
+#define COSPEC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(_WIN32)
+#define COSPEC_API
+#else
+#define COSPEC_API __attribute__((visibility("default")))
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  COSPEC_OK = 0,
+  COSPEC_ERR_INVALID_ARG = -1,  /* null pointer, bad size or inconsistent shape */
+  COSPEC_ERR_UNSUPPORTED = -2,  /* valid but outside the shapes the kernels handle */
+  COSPEC_ERR_WORKSPACE = -3,    /* workspace missing or smaller than required */
+  COSPEC_ERR_CUDA = -4,         /* a CUDA runtime call or a launch failed */
+  COSPEC_ERR_DEVICE_CHECK = -5  /* the device error word was non-zero */
+} cospec_status;
+
+/* Bits of the device error word. */
+#define COSPEC_DEVERR_PAGE 1     /* page id outside [0, num_pages) */
+#define COSPEC_DEVERR_CTX 2      /* ctx_len < 0, ctx_len > max_ctx (attention), or ctx_len plus the
+                                    accepted rows > max_pages_per_seq * page_size (commit) */
+#define COSPEC_DEVERR_TOKEN 4    /* token id outside the vocabulary */
+#define COSPEC_DEVERR_TIMEOUT 8  /* a bounded pipeline wait gave up (never expected) */
+
+/* Human-readable name of a cospec_status value (static string). */
+COSPEC_API const char* cospec_status_string(int status);
+
+/* Reads the device error word into *flags, then clears it.  Synchronises
+ * `stream` first, so every kernel queued before is included.  Returns
+ * COSPEC_OK, or COSPEC_ERR_DEVICE_CHECK when *flags != 0. */
+COSPEC_API int cospec_get_device_error(int* flags, void* stream);
+
+/* Number of SMs of the current device (used to size grids; cached). */
+COSPEC_API int cospec_num_sms(void);
+
+/* ------------------------------------------------------------------------ */
+/* 1. Verify attention (Sec. 3.1, Eq. 2: one teacher-forced pass of the
+ *    target over [x, y^(<r), y_hat_1..y_hat_K]; this call is the attention
+ *    of one layer of that pass for the K+1 rightmost positions).
+ *
+ *    For sequence b, query head h, block row j:
+ *      o = softmax(q . k^T * softmax_scale + mask) . v
+ *    over the ctx_len[b] committed positions of the paged cache followed by
+ *    block rows 0..j of (k_blk, v_blk) (causal inside the block).  Query
+ *    head h reads KV head h / (num_q_heads / num_kv_heads) (GQA).
+ *
+ *    q        bf16 [batch, rows, num_q_heads, head_dim]
+ *    k_blk    bf16 [batch, rows, num_kv_heads, head_dim]   this layer's block keys
+ *    v_blk    bf16 [batch, rows, num_kv_heads, head_dim]
+ *    k_pages  bf16 [num_pages, num_kv_heads, page_size, head_dim]   this layer's pool
+ *    v_pages  bf16 [num_pages, num_kv_heads, page_size, head_dim]
+ *    page_table int32 [batch, max_pages_per_seq]: logical page p of sequence b
+ *             is physical page page_table[b * max_pages_per_seq + p]; only the
+ *             first ceil(ctx_len[b] / page_size) entries are read.
+ *    ctx_len  int32 [batch]
+ *    out      bf16 [batch, rows, num_q_heads, head_dim] (may not alias inputs)
+ *    max_ctx  an upper bound of ctx_len[*] (host-side; sizes the KV split)
+ *    ws       device workspace of at least cospec_verify_attn_workspace()
+ *             bytes.  Its first cospec_verify_attn_ticket_bytes() bytes are
+ *             split counters that must be zero before the first call
+ *             (cudaMemset once); every completed call leaves them zero.
+ *             Calls that run concurrently need distinct workspaces.
+ *    Supported: head_dim in {64, 128}; page_size == 16; rows <= 32;
+ *    num_q_heads % num_kv_heads == 0; (num_q_heads / num_kv_heads) * rows <= 128.
+ * ------------------------------------------------------------------------ */
+typedef struct {
+  int batch;
+  int rows;              /* R = K + 1 */
+  int num_q_heads;
+  int num_kv_heads;
+  int head_dim;
+  int page_size;
+  int max_pages_per_seq;
+  int num_pages;
+  float softmax_scale;   /* <= 0 selects 1/sqrt(head_dim) */
+} cospec_attn_dims;
+
+COSPEC_API size_t cospec_verify_attn_workspace(const cospec_attn_dims* dims, int max_ctx);
+COSPEC_API size_t cospec_verify_attn_ticket_bytes(const cospec_attn_dims* dims);
+COSPEC_API int cospec_verify_attn(const cospec_attn_dims* dims, int max_ctx,
+                                  const uint16_t* q, const uint16_t* k_blk, const uint16_t* v_blk,
+                                  const uint16_t* k_pages, const uint16_t* v_pages,
+                                  const int32_t* page_table, const int32_t* ctx_len,
+                                  uint16_t* out, void* ws, size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------ */
+/* 2. LM head fused with argmax and log-prob statistics (Eq. 2 gives the
+ *    target prediction y_tilde = argmax of each row's logits; Eq. 23 defines
+ *    l_i = log p_T(y_hat_i | prefix) = x[y_hat_i] - lse).
+ *
+ *    For each of the M rows: x = hidden[m] . W^T (fp32 accumulation of bf16
+ *    products; the M x V logits are never written to memory) and
+ *      argmax[m]   = lowest id among the maximal logits (y_tilde)
+ *      stats[m][0] = max_v x_v
+ *      stats[m][1] = largest logit over ids != argmax (equals [0] on a tie)
+ *      stats[m][2] = lse = log sum_v exp(x_v)
+ *      stats[m][3] = entropy = lse - sum_v softmax(x)_v x_v
+ *      stats[m][4] = x[draft_for_row[m]], NaN when draft_for_row[m] == -1
+ *
+ *    hidden   bf16 [M, d];  w  bf16 [V, d] (nn.Linear weight layout)
+ *    draft_for_row int32 [M] in [-1, V): the draft id scored by row m
+ *    argmax   int32 [M];  stats float32 [M, 5]
+ *    ws       >= cospec_lmhead_workspace(M, d, V) bytes (no initialisation)
+ *    Supported: d % 64 == 0, 1 <= M, V >= 1; hidden and w 16-byte aligned.
+ *    Runs on tcgen05 tensor cores (TMEM accumulators, TMA-fed operands).
+ * ------------------------------------------------------------------------ */
+COSPEC_API size_t cospec_lmhead_workspace(int M, int d, int V);
+COSPEC_API int cospec_lmhead_argmax_features(int M, int d, int V, const uint16_t* hidden,
+                                             const uint16_t* w, const int32_t* draft_for_row,
+                                             int32_t* argmax, float* stats, void* ws,
+                                             size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------ */
+/* 3. Arbitration at draft/target mismatches (Sec. 3.3).
+ *
+ *    Delta_i = 1[draft[b,i-1] == argmax[b,i-1]] (Eq. 3).  Matches are forced
+ *    accepted: p = sigma(+inf) = 1, accept = 1 (Eq. 13-14).  At a mismatch
+ *    p = sigma(z) with z = w2 . ReLU(W1 f_i + b1) + b2 for policy_mode 0,
+ *    p = 0 for policy_mode 1 ("always target", exact-match decoding) and
+ *    p = 1 for policy_mode 2 ("always draft"); accept = 1[p > lambda]
+ *    (Eq. 17, strict).  f_i is the 8-feature vector built from the target
+ *    statistics of rows i-1 and i (F0 = x_{i-1}[y_hat_i] - lse_{i-1},
+ *    F1 = max_{i-1} - lse_{i-1}, F2 = max_{i-1} - second_{i-1},
+ *    F3 = entropy_{i-1}, F4 = max_i - lse_i, F5 = x_i[y_hat_{i+1}] - lse_i
+ *    (0 at i = K), F6 = i/K, F7 = #{j < i : Delta_j = 1}/K).
+ *
+ *    draft  int32 [B, K];  argmax int32 [B, K+1];  stats float32 [B, K+1, 5]
+ *    w1 float32 [mlp_hidden, 8], b1 [mlp_hidden], w2 [mlp_hidden] (device;
+ *    may be NULL when policy_mode != 0);  p_out float32 [B, K];
+ *    accept uint8 [B, K].  Supported: 0 <= K <= 31, mlp_hidden <= 1024.
+ * ------------------------------------------------------------------------ */
+#define COSPEC_POLICY_MLP 0
+#define COSPEC_POLICY_TARGET 1
+#define COSPEC_POLICY_DRAFT 2
+
+COSPEC_API int cospec_arbitrate(int B, int K, const int32_t* draft, const int32_t* argmax,
+                                const float* stats, int mlp_hidden, const float* w1,
+                                const float* b1, const float* w2, float b2, float lambda,
+                                int policy_mode, float* p_out, uint8_t* accept, void* stream);
+
+/* ------------------------------------------------------------------------ */
+/* 4. Accepted length, emitted tokens and KV commit (Eq. 15; App. F).
+ *
+ *    s_b = min{i : Delta_i = 0 and accept_i = 0}, else K+1.  The round emits
+ *    draft_1..draft_{s-1} followed by argmax row s-1 (y_tilde_s; the bonus
+ *    when s = K+1).  Block rows 0..s-1 of every layer's staging K/V are then
+ *    copied to cache positions ctx_len[b] .. ctx_len[b]+s-1 through the page
+ *    table, and ctx_len[b] += s.  Rows after s never reach the cache.
+ *
+ *    draft int32 [B, K]; argmax int32 [B, K+1]; accept uint8 [B, K]
+ *    k_blk, v_blk  bf16 [num_layers, B, K+1, num_kv_heads, head_dim]
+ *    k_pages, v_pages  bf16: layer l's pool [num_pages, num_kv_heads,
+ *             page_size, head_dim] starts pool_layer_stride elements after
+ *             layer l-1's (pool_layer_stride >= num_pages*Hkv*P*D, or 0 when
+ *             every layer shares one pool)
+ *    dims     the attention geometry (batch == B, rows == K+1)
+ *    ctx_len  int32 [B], updated in place
+ *    accept_len int32 [B]; emitted int32 [B, K+1] (padded with -1)
+ * ------------------------------------------------------------------------ */
+COSPEC_API int cospec_accept_commit(int B, int K, int num_layers, const cospec_attn_dims* dims,
+                                    const int32_t* draft, const int32_t* argmax,
+                                    const uint8_t* accept, const uint16_t* k_blk,
+                                    const uint16_t* v_blk, uint16_t* k_pages, uint16_t* v_pages,
+                                    long long pool_layer_stride, const int32_t* page_table,
+                                    int32_t* ctx_len, int32_t* accept_len, int32_t* emitted,
+                                    void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* COSPEC_H */

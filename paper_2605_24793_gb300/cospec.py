@@ -1,0 +1,238 @@
+"""Python binding of libcospec.so: the same four calls as include/cospec.h.
+
+Argument marshalling only -- shapes are read off the tensors, pointers and
+the current CUDA stream are passed through ctypes, and every step runs in
+the library's CUDA kernels.  There is no CPU or PyTorch fallback: if the
+library is missing or a call fails, an exception is raised.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libcospec.so")
+
+POLICY_MLP, POLICY_TARGET, POLICY_DRAFT = 0, 1, 2
+DEVERR_PAGE, DEVERR_CTX, DEVERR_TOKEN, DEVERR_TIMEOUT = 1, 2, 4, 8
+
+EXPORTED = ("cospec_status_string", "cospec_get_device_error", "cospec_num_sms",
+            "cospec_verify_attn_workspace", "cospec_verify_attn_ticket_bytes",
+            "cospec_verify_attn", "cospec_lmhead_workspace", "cospec_lmhead_argmax_features",
+            "cospec_arbitrate", "cospec_accept_commit")
+
+
+class AttnDims(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int), ("rows", ctypes.c_int), ("num_q_heads", ctypes.c_int),
+                ("num_kv_heads", ctypes.c_int), ("head_dim", ctypes.c_int),
+                ("page_size", ctypes.c_int), ("max_pages_per_seq", ctypes.c_int),
+                ("num_pages", ctypes.c_int), ("softmax_scale", ctypes.c_float)]
+
+
+class CospecError(RuntimeError):
+    pass
+
+
+_lib: Optional[ctypes.CDLL] = None
+
+_vp, _i, _sz, _f = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t, ctypes.c_float
+_PDIMS = ctypes.POINTER(AttnDims)
+
+
+def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Load libcospec.so (built by ``paper_2605_24793_gb300.build``)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise CospecError(f"{path} is missing; build it with python -m paper_2605_24793_gb300.build")
+    lib = ctypes.CDLL(path)
+    sig = {
+        "cospec_status_string": (ctypes.c_char_p, [_i]),
+        "cospec_get_device_error": (_i, [ctypes.POINTER(_i), _vp]),
+        "cospec_num_sms": (_i, []),
+        "cospec_verify_attn_workspace": (_sz, [_PDIMS, _i]),
+        "cospec_verify_attn_ticket_bytes": (_sz, [_PDIMS]),
+        "cospec_verify_attn": (_i, [_PDIMS, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+        "cospec_lmhead_workspace": (_sz, [_i, _i, _i]),
+        "cospec_lmhead_argmax_features": (_i, [_i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+        "cospec_arbitrate": (_i, [_i, _i, _vp, _vp, _vp, _i, _vp, _vp, _vp, _f, _f, _i, _vp, _vp, _vp]),
+        "cospec_accept_commit": (_i, [_i, _i, _i, _PDIMS, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                      ctypes.c_longlong, _vp, _vp, _vp, _vp, _vp]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _check(status: int) -> None:
+    if status != 0:
+        msg = load_library().cospec_status_string(status).decode()
+        raise CospecError(f"cospec call failed: {msg} ({status})")
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _req(t: torch.Tensor, dtype, name: str, ndim: Optional[int] = None):
+    if t.dtype != dtype:
+        raise TypeError(f"{name}: expected {dtype}, got {t.dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name}: must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name}: must be contiguous")
+    if ndim is not None and t.dim() != ndim:
+        raise ValueError(f"{name}: expected {ndim} dims, got {t.dim()}")
+
+
+def attn_dims(q: torch.Tensor, k_pages: torch.Tensor, page_table: torch.Tensor,
+              softmax_scale: float = 0.0) -> AttnDims:
+    """Geometry of one verify-attention call from q [B,R,Hq,D], the layer's
+    pool [num_pages,Hkv,P,D] and the page table [B,max_pages]."""
+    B, R, Hq, D = q.shape
+    num_pages, Hkv, P, D2 = k_pages.shape[-4:]
+    assert D2 == D
+    return AttnDims(B, R, Hq, Hkv, D, P, page_table.shape[1], num_pages, softmax_scale)
+
+
+def num_sms() -> int:
+    return load_library().cospec_num_sms()
+
+
+def verify_attn_workspace_bytes(dims: AttnDims, max_ctx: int) -> int:
+    return load_library().cospec_verify_attn_workspace(ctypes.byref(dims), max_ctx)
+
+
+def new_attn_workspace(dims: AttnDims, max_ctx: int, device="cuda") -> torch.Tensor:
+    """Workspace for cospec_verify_attn, zeroed (its split counters must start at 0)."""
+    n = verify_attn_workspace_bytes(dims, max_ctx)
+    if n == 0:
+        raise CospecError("unsupported attention geometry")
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def verify_attn(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len, out, ws, max_ctx,
+                softmax_scale: float = 0.0, stream=None) -> torch.Tensor:
+    """Verify attention of one layer (Sec. 3.1, Eq. 2).  See include/cospec.h."""
+    for t, n in ((q, "q"), (k_blk, "k_blk"), (v_blk, "v_blk"), (k_pages, "k_pages"),
+                 (v_pages, "v_pages"), (out, "out")):
+        _req(t, torch.bfloat16, n)
+    _req(page_table, torch.int32, "page_table", 2)
+    _req(ctx_len, torch.int32, "ctx_len", 1)
+    _req(ws, torch.uint8, "ws", 1)
+    dims = attn_dims(q, k_pages, page_table, softmax_scale)
+    if tuple(k_blk.shape) != (dims.batch, dims.rows, dims.num_kv_heads, dims.head_dim):
+        raise ValueError("k_blk shape does not match q / pages")
+    if out.shape != q.shape:
+        raise ValueError("out must have q's shape")
+    _check(load_library().cospec_verify_attn(
+        ctypes.byref(dims), int(max_ctx), _ptr(q), _ptr(k_blk), _ptr(v_blk), _ptr(k_pages),
+        _ptr(v_pages), _ptr(page_table), _ptr(ctx_len), _ptr(out), _ptr(ws), ws.numel(),
+        _stream(stream)))
+    return out
+
+
+def lmhead_workspace_bytes(M: int, d: int, V: int) -> int:
+    return load_library().cospec_lmhead_workspace(M, d, V)
+
+
+def new_lmhead_workspace(M: int, d: int, V: int, device="cuda") -> torch.Tensor:
+    return torch.empty(lmhead_workspace_bytes(M, d, V), dtype=torch.uint8, device=device)
+
+
+def lmhead_argmax_features(hidden, w, draft_for_row, argmax, stats, ws, stream=None):
+    """LM head + argmax + statistics (Eq. 2, Eq. 23).  stats [M,5] = (max,
+    second, lse, entropy, draft logit)."""
+    _req(hidden, torch.bfloat16, "hidden", 2)
+    _req(w, torch.bfloat16, "w", 2)
+    _req(draft_for_row, torch.int32, "draft_for_row", 1)
+    _req(argmax, torch.int32, "argmax", 1)
+    _req(stats, torch.float32, "stats", 2)
+    _req(ws, torch.uint8, "ws", 1)
+    M, d = hidden.shape
+    V = w.shape[0]
+    if w.shape[1] != d or draft_for_row.numel() != M or argmax.numel() != M or tuple(stats.shape) != (M, 5):
+        raise ValueError("inconsistent LM-head shapes")
+    _check(load_library().cospec_lmhead_argmax_features(
+        M, d, V, _ptr(hidden), _ptr(w), _ptr(draft_for_row), _ptr(argmax), _ptr(stats), _ptr(ws),
+        ws.numel(), _stream(stream)))
+    return argmax, stats
+
+
+def arbitrate(draft, argmax, stats, w1, b1, w2, b2: float, lam: float, mode: int, p_out, accept,
+              stream=None):
+    """Mismatch arbitration (Eq. 3, Eq. 13-14, Eq. 17).  draft [B,K],
+    argmax [B,K+1], stats [B,K+1,5]; p_out [B,K] float32, accept [B,K] uint8."""
+    _req(draft, torch.int32, "draft", 2)
+    _req(argmax, torch.int32, "argmax")
+    _req(stats, torch.float32, "stats")
+    _req(p_out, torch.float32, "p_out")
+    _req(accept, torch.uint8, "accept")
+    B, K = draft.shape
+    if argmax.numel() != B * (K + 1) or stats.numel() != B * (K + 1) * 5:
+        raise ValueError("argmax / stats must hold K+1 rows per sequence")
+    H = 0
+    if mode == POLICY_MLP:
+        for t, n in ((w1, "w1"), (b1, "b1"), (w2, "w2")):
+            _req(t, torch.float32, n)
+        H = w1.shape[0]
+    _check(load_library().cospec_arbitrate(
+        B, K, _ptr(draft), _ptr(argmax), _ptr(stats), H, _ptr(w1) if mode == 0 else None,
+        _ptr(b1) if mode == 0 else None, _ptr(w2) if mode == 0 else None, float(b2), float(lam),
+        int(mode), _ptr(p_out), _ptr(accept), _stream(stream)))
+    return p_out, accept
+
+
+def accept_commit(draft, argmax, accept, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len,
+                  accept_len, emitted, stream=None):
+    """Accepted length / emitted tokens (Eq. 15) and KV commit.
+    k_blk, v_blk [L,B,R,Hkv,D]; pools [L,num_pages,Hkv,P,D] (any layer stride)."""
+    _req(draft, torch.int32, "draft", 2)
+    _req(argmax, torch.int32, "argmax")
+    _req(accept, torch.uint8, "accept")
+    for t, n in ((k_blk, "k_blk"), (v_blk, "v_blk")):
+        _req(t, torch.bfloat16, n, 5)
+    for t, n in ((k_pages, "k_pages"), (v_pages, "v_pages")):
+        if t.dtype != torch.bfloat16 or not t.is_cuda or t.dim() != 5 or not t[0].is_contiguous():
+            raise ValueError(f"{n}: expected bf16 CUDA [L,num_pages,Hkv,P,D] with contiguous layers")
+    _req(page_table, torch.int32, "page_table", 2)
+    _req(ctx_len, torch.int32, "ctx_len", 1)
+    _req(accept_len, torch.int32, "accept_len", 1)
+    _req(emitted, torch.int32, "emitted")
+    B, K = draft.shape
+    L = k_blk.shape[0]
+    if k_pages.shape[0] not in (L, 1) or k_pages.shape != v_pages.shape or \
+            k_pages.stride(0) != v_pages.stride(0):
+        raise ValueError("k_pages / v_pages must hold the same layers with the same stride")
+    # a single pool shared by every layer is passed with layer stride 0
+    layer_stride = 0 if (k_pages.shape[0] == 1 and L > 1) else int(k_pages.stride(0))
+    dims = AttnDims(B, K + 1, 0, k_pages.shape[2], k_pages.shape[4], k_pages.shape[3],
+                    page_table.shape[1], k_pages.shape[1], 0.0)
+    dims.num_q_heads = dims.num_kv_heads
+    _check(load_library().cospec_accept_commit(
+        B, K, L, ctypes.byref(dims), _ptr(draft), _ptr(argmax), _ptr(accept), _ptr(k_blk),
+        _ptr(v_blk), _ptr(k_pages), _ptr(v_pages), layer_stride, _ptr(page_table),
+        _ptr(ctx_len), _ptr(accept_len), _ptr(emitted), _stream(stream)))
+    return accept_len, emitted
+
+
+def get_device_error(stream=None) -> int:
+    """Read and clear the device error word (synchronises the stream)."""
+    flags = ctypes.c_int(0)
+    st = load_library().cospec_get_device_error(ctypes.byref(flags), _stream(stream))
+    if st not in (0, -5):
+        _check(st)
+    return flags.value

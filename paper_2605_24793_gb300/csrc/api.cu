@@ -1,0 +1,259 @@
+// C ABI of the verify/arbitrate round: host-side validation, workspace
+// sizing, the device error word and dispatch to the kernel launchers.
+#include <math.h>
+#include <stdint.h>
+
+#include "../../include/cospec.h"
+#include "cospec_internal.h"
+
+namespace cospec {
+
+namespace {
+__device__ int g_error_word;   // one per device context; bits COSPEC_DEVERR_*
+
+constexpr int MAX_DEV = 64;
+int g_num_sms[MAX_DEV] = {0};
+int* g_err_ptr[MAX_DEV] = {nullptr};
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int current_device() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return -1;
+  return dev;
+}
+}  // namespace
+
+int device_num_sms() {
+  const int dev = current_device();
+  if (dev < 0 || dev >= MAX_DEV) return 0;
+  if (g_num_sms[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    g_num_sms[dev] = n;
+  }
+  return g_num_sms[dev];
+}
+
+int* device_error_word() {
+  const int dev = current_device();
+  if (dev < 0 || dev >= MAX_DEV) return nullptr;
+  if (!g_err_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
+    g_err_ptr[dev] = static_cast<int*>(p);
+  }
+  return g_err_ptr[dev];
+}
+
+}  // namespace cospec
+
+using namespace cospec;
+
+#define CS_CHECK_ARG(cond)                 \
+  do {                                     \
+    if (!(cond)) return COSPEC_ERR_INVALID_ARG; \
+  } while (0)
+
+static int from_cuda(cudaError_t e) { return e == cudaSuccess ? COSPEC_OK : COSPEC_ERR_CUDA; }
+
+extern "C" {
+
+COSPEC_API const char* cospec_status_string(int status) {
+  switch (status) {
+    case COSPEC_OK: return "ok";
+    case COSPEC_ERR_INVALID_ARG: return "invalid argument";
+    case COSPEC_ERR_UNSUPPORTED: return "unsupported shape";
+    case COSPEC_ERR_WORKSPACE: return "workspace missing or too small";
+    case COSPEC_ERR_CUDA: return "CUDA runtime error";
+    case COSPEC_ERR_DEVICE_CHECK: return "device-side check failed";
+    default: return "unknown status";
+  }
+}
+
+COSPEC_API int cospec_num_sms(void) { return device_num_sms(); }
+
+COSPEC_API int cospec_get_device_error(int* flags, void* stream) {
+  CS_CHECK_ARG(flags != nullptr);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int* dptr = device_error_word();
+  if (!dptr) return COSPEC_ERR_CUDA;
+  int v = 0;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return COSPEC_ERR_CUDA;
+  if (cudaMemcpyAsync(&v, dptr, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess)
+    return COSPEC_ERR_CUDA;
+  if (cudaMemsetAsync(dptr, 0, sizeof(int), st) != cudaSuccess) return COSPEC_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return COSPEC_ERR_CUDA;
+  *flags = v;
+  return v ? COSPEC_ERR_DEVICE_CHECK : COSPEC_OK;
+}
+
+// ---------------------------------------------------------------- attention
+static int check_attn_dims(const cospec_attn_dims* d) {
+  if (!d) return COSPEC_ERR_INVALID_ARG;
+  if (d->batch < 0 || d->rows < 1 || d->num_q_heads < 1 || d->num_kv_heads < 1 ||
+      d->head_dim < 1 || d->page_size < 1 || d->max_pages_per_seq < 1 || d->num_pages < 1)
+    return COSPEC_ERR_INVALID_ARG;
+  if (d->num_q_heads % d->num_kv_heads != 0) return COSPEC_ERR_INVALID_ARG;
+  if (isnan(d->softmax_scale) || isinf(d->softmax_scale)) return COSPEC_ERR_INVALID_ARG;
+  if (d->head_dim != 64 && d->head_dim != 128) return COSPEC_ERR_UNSUPPORTED;
+  if (d->page_size != 16) return COSPEC_ERR_UNSUPPORTED;
+  if (d->rows > 32) return COSPEC_ERR_UNSUPPORTED;
+  if ((d->num_q_heads / d->num_kv_heads) * d->rows > 128) return COSPEC_ERR_UNSUPPORTED;
+  return COSPEC_OK;
+}
+
+COSPEC_API size_t cospec_verify_attn_workspace(const cospec_attn_dims* d, int max_ctx) {
+  if (check_attn_dims(d) != COSPEC_OK || max_ctx < 0) return 0;
+  const int sms = device_num_sms();
+  const AttnPlan pl = plan_verify_attn(d->batch, d->rows, d->num_q_heads, d->num_kv_heads,
+                                       d->head_dim, max_ctx, sms > 0 ? sms : 148);
+  return pl.total_bytes;
+}
+
+COSPEC_API size_t cospec_verify_attn_ticket_bytes(const cospec_attn_dims* d) {
+  if (check_attn_dims(d) != COSPEC_OK) return 0;
+  return (((size_t)d->batch * d->num_kv_heads * sizeof(int)) + 255) / 256 * 256;
+}
+
+COSPEC_API int cospec_verify_attn(const cospec_attn_dims* d, int max_ctx, const uint16_t* q,
+                                  const uint16_t* k_blk, const uint16_t* v_blk,
+                                  const uint16_t* k_pages, const uint16_t* v_pages,
+                                  const int32_t* page_table, const int32_t* ctx_len, uint16_t* out,
+                                  void* ws, size_t ws_bytes, void* stream) {
+  const int st = check_attn_dims(d);
+  if (st != COSPEC_OK) return st;
+  CS_CHECK_ARG(max_ctx >= 0 && max_ctx <= d->max_pages_per_seq * d->page_size);
+  if (d->batch == 0) return COSPEC_OK;
+  CS_CHECK_ARG(q && k_blk && v_blk && k_pages && v_pages && page_table && ctx_len && out);
+  CS_CHECK_ARG(aligned16(q) && aligned16(k_blk) && aligned16(v_blk) && aligned16(k_pages) &&
+               aligned16(v_pages) && aligned16(out));
+  const int sms = device_num_sms();
+  if (sms <= 0) return COSPEC_ERR_CUDA;
+  const AttnPlan pl = plan_verify_attn(d->batch, d->rows, d->num_q_heads, d->num_kv_heads,
+                                       d->head_dim, max_ctx, sms);
+  if (!ws || ws_bytes < pl.total_bytes || !aligned16(ws)) return COSPEC_ERR_WORKSPACE;
+  int* err = device_error_word();
+  if (!err) return COSPEC_ERR_CUDA;
+  AttnArgs a{};
+  a.q = reinterpret_cast<const __nv_bfloat16*>(q);
+  a.k_blk = reinterpret_cast<const __nv_bfloat16*>(k_blk);
+  a.v_blk = reinterpret_cast<const __nv_bfloat16*>(v_blk);
+  a.k_pages = reinterpret_cast<const __nv_bfloat16*>(k_pages);
+  a.v_pages = reinterpret_cast<const __nv_bfloat16*>(v_pages);
+  a.page_table = page_table;
+  a.ctx_len = ctx_len;
+  a.out = reinterpret_cast<__nv_bfloat16*>(out);
+  a.B = d->batch;
+  a.R = d->rows;
+  a.Hq = d->num_q_heads;
+  a.Hkv = d->num_kv_heads;
+  a.D = d->head_dim;
+  a.P = d->page_size;
+  a.max_pages = d->max_pages_per_seq;
+  a.num_pages = d->num_pages;
+  a.scale = d->softmax_scale > 0.f ? d->softmax_scale : 1.0f / sqrtf((float)d->head_dim);
+  a.max_ctx = max_ctx;
+  a.ws = ws;
+  a.ws_bytes = ws_bytes;
+  return from_cuda(launch_verify_attn(a, pl, err, static_cast<cudaStream_t>(stream)));
+}
+
+// ---------------------------------------------------------------- LM head
+COSPEC_API size_t cospec_lmhead_workspace(int M, int d, int V) {
+  if (M < 1 || d < 64 || V < 1) return 0;
+  const int sms = device_num_sms();
+  return plan_lmhead(M, d, V, sms > 0 ? sms : 148).ws_bytes;
+}
+
+COSPEC_API int cospec_lmhead_argmax_features(int M, int d, int V, const uint16_t* hidden,
+                                             const uint16_t* w, const int32_t* draft_for_row,
+                                             int32_t* argmax, float* stats, void* ws,
+                                             size_t ws_bytes, void* stream) {
+  CS_CHECK_ARG(M >= 0 && d > 0 && V > 0);
+  if (M == 0) return COSPEC_OK;
+  CS_CHECK_ARG(hidden && w && draft_for_row && argmax && stats);
+  if (d % 64 != 0) return COSPEC_ERR_UNSUPPORTED;
+  if ((long long)V > 0x7fffff00LL) return COSPEC_ERR_UNSUPPORTED;
+  CS_CHECK_ARG(aligned16(hidden) && aligned16(w));
+  const int sms = device_num_sms();
+  if (sms <= 0) return COSPEC_ERR_CUDA;
+  const LmheadPlan pl = plan_lmhead(M, d, V, sms);
+  if (!ws || ws_bytes < pl.ws_bytes || !aligned16(ws)) return COSPEC_ERR_WORKSPACE;
+  int* err = device_error_word();
+  if (!err) return COSPEC_ERR_CUDA;
+  return from_cuda(launch_lmhead(M, d, V, reinterpret_cast<const __nv_bfloat16*>(hidden),
+                                 reinterpret_cast<const __nv_bfloat16*>(w), draft_for_row, argmax,
+                                 stats, ws, pl, err, static_cast<cudaStream_t>(stream)));
+}
+
+// ---------------------------------------------------------------- arbitration
+COSPEC_API int cospec_arbitrate(int B, int K, const int32_t* draft, const int32_t* argmax,
+                                const float* stats, int mlp_hidden, const float* w1,
+                                const float* b1, const float* w2, float b2, float lambda,
+                                int policy_mode, float* p_out, uint8_t* accept, void* stream) {
+  CS_CHECK_ARG(B >= 0 && K >= 0);
+  if (K > 31) return COSPEC_ERR_UNSUPPORTED;
+  CS_CHECK_ARG(policy_mode >= 0 && policy_mode <= 2);
+  CS_CHECK_ARG(!isnan(lambda));
+  if (B == 0 || K == 0) return COSPEC_OK;
+  CS_CHECK_ARG(draft && argmax && stats && p_out && accept);
+  if (policy_mode == COSPEC_POLICY_MLP) {
+    CS_CHECK_ARG(w1 && b1 && w2 && mlp_hidden >= 1 && !isnan(b2));
+    if (mlp_hidden > 1024) return COSPEC_ERR_UNSUPPORTED;
+  }
+  return from_cuda(launch_arbitrate(B, K, draft, argmax, stats, mlp_hidden, w1, b1, w2, b2, lambda,
+                                    policy_mode, p_out, accept, static_cast<cudaStream_t>(stream)));
+}
+
+// ---------------------------------------------------------------- accept + commit
+COSPEC_API int cospec_accept_commit(int B, int K, int num_layers, const cospec_attn_dims* dims,
+                                    const int32_t* draft, const int32_t* argmax,
+                                    const uint8_t* accept, const uint16_t* k_blk,
+                                    const uint16_t* v_blk, uint16_t* k_pages, uint16_t* v_pages,
+                                    long long pool_layer_stride, const int32_t* page_table,
+                                    int32_t* ctx_len, int32_t* accept_len, int32_t* emitted,
+                                    void* stream) {
+  CS_CHECK_ARG(B >= 0 && K >= 0 && num_layers >= 0);
+  if (K > 31) return COSPEC_ERR_UNSUPPORTED;
+  const int st = check_attn_dims(dims);
+  if (st != COSPEC_OK) return st;
+  CS_CHECK_ARG(dims->batch == B && dims->rows == K + 1);
+  if (B == 0) return COSPEC_OK;
+  CS_CHECK_ARG(argmax && ctx_len && accept_len && emitted && page_table);
+  CS_CHECK_ARG(K == 0 || (draft && accept));
+  const long long pool_elems = (long long)dims->num_pages * dims->num_kv_heads * dims->page_size *
+                               dims->head_dim;
+  if (num_layers > 0) {
+    CS_CHECK_ARG(k_blk && v_blk && k_pages && v_pages);
+    CS_CHECK_ARG(aligned16(k_blk) && aligned16(v_blk) && aligned16(k_pages) && aligned16(v_pages));
+    CS_CHECK_ARG(num_layers == 1 || pool_layer_stride == 0 || pool_layer_stride >= pool_elems);
+    CS_CHECK_ARG(pool_layer_stride % 8 == 0);
+  }
+  int* err = device_error_word();
+  if (!err) return COSPEC_ERR_CUDA;
+  CommitArgs a{};
+  a.B = B;
+  a.K = K;
+  a.L = num_layers;
+  a.Hkv = dims->num_kv_heads;
+  a.D = dims->head_dim;
+  a.P = dims->page_size;
+  a.max_pages = dims->max_pages_per_seq;
+  a.num_pages = dims->num_pages;
+  a.pool_layer_stride = pool_layer_stride;
+  a.draft = draft;
+  a.argmax = argmax;
+  a.accept = accept;
+  a.k_blk = reinterpret_cast<const __nv_bfloat16*>(k_blk);
+  a.v_blk = reinterpret_cast<const __nv_bfloat16*>(v_blk);
+  a.k_pages = reinterpret_cast<__nv_bfloat16*>(k_pages);
+  a.v_pages = reinterpret_cast<__nv_bfloat16*>(v_pages);
+  a.page_table = page_table;
+  a.ctx_len = ctx_len;
+  a.accept_len = accept_len;
+  a.emitted = emitted;
+  return from_cuda(launch_accept_commit(a, err, static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

@@ -1,0 +1,79 @@
+// Internal host-side interface between the C-ABI layer (api.cu) and the
+// kernel translation units.  Not part of the public ABI.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace cospec {
+
+int device_num_sms();
+int* device_error_word();  // device address of the error word of the current device
+
+// ---------------------------------------------------------------- attention
+struct AttnArgs {
+  const __nv_bfloat16* q;
+  const __nv_bfloat16* k_blk;
+  const __nv_bfloat16* v_blk;
+  const __nv_bfloat16* k_pages;
+  const __nv_bfloat16* v_pages;
+  const int32_t* page_table;
+  const int32_t* ctx_len;
+  __nv_bfloat16* out;
+  int B, R, Hq, Hkv, D, P, max_pages, num_pages;
+  float scale;
+  int max_ctx;
+  void* ws;
+  size_t ws_bytes;
+};
+struct AttnPlan {
+  int mt, wk, tiles_per_split, max_splits, nrp;
+  size_t ticket_bytes, partial_bytes, ml_bytes, total_bytes;
+};
+AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int num_sms);
+cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& plan, int* err,
+                               cudaStream_t stream);
+
+// ---------------------------------------------------------------- LM head
+struct LmheadPlan {
+  int n_mma;       // MMA N (padded rows per pass), multiple of 16, <= 256
+  int passes;      // ceil(M / 256)
+  int num_tiles;   // ceil(V / 128)
+  int grid;        // persistent CTAs
+  int stages;
+  size_t smem_bytes;
+  size_t ws_bytes;
+};
+LmheadPlan plan_lmhead(int M, int d, int V, int num_sms);
+cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
+                          const __nv_bfloat16* w, const int32_t* draft_for_row, int32_t* argmax,
+                          float* stats, void* ws, const LmheadPlan& plan, int* err,
+                          cudaStream_t stream);
+
+// ---------------------------------------------------------------- arbitration
+cudaError_t launch_arbitrate(int B, int K, const int32_t* draft, const int32_t* argmax,
+                             const float* stats, int H, const float* w1, const float* b1,
+                             const float* w2, float b2, float lambda, int mode, float* p_out,
+                             uint8_t* accept, cudaStream_t stream);
+
+// ---------------------------------------------------------------- accept + commit
+struct CommitArgs {
+  int B, K, L, Hkv, D, P, max_pages, num_pages;
+  long long pool_layer_stride;
+  const int32_t* draft;
+  const int32_t* argmax;
+  const uint8_t* accept;
+  const __nv_bfloat16* k_blk;
+  const __nv_bfloat16* v_blk;
+  __nv_bfloat16* k_pages;
+  __nv_bfloat16* v_pages;
+  const int32_t* page_table;
+  int32_t* ctx_len;
+  int32_t* accept_len;
+  int32_t* emitted;
+};
+cudaError_t launch_accept_commit(const CommitArgs& a, int* err, cudaStream_t stream);
+
+}  // namespace cospec

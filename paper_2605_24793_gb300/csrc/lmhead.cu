@@ -1,0 +1,502 @@
+// LM head fused with argmax and log-prob statistics (Sec. 3.1 Eq. 2: the
+// target prediction y_tilde is the argmax of each block row's logits;
+// Eq. 23: l_i = x[y_hat_i] - lse).  The M x V logits never reach memory.
+//
+// tcgen05 swap-AB GEMM: the vocabulary is the MMA M dimension (128 rows of W
+// per tile) and the verify rows are N (padded to a multiple of 16, <= 256 per
+// pass), so a handful of rows still fills the tensor core and W -- the only
+// large operand -- is streamed from HBM exactly once.  Persistent CTAs (one
+// per SM) walk vocabulary tiles; warp 0 issues TMA loads (128B swizzle, W
+// with evict-first, hidden rows with evict-last) into a ring of stages,
+// warp 1 issues tcgen05.mma into one of two TMEM accumulators, warps 2-5 read
+// the finished accumulator with tcgen05.ld and fold it into per-row running
+// statistics while the next tile is multiplied.  A second small kernel
+// merges the per-CTA partials.
+//
+// Statistics are kept as a tuple (m, i, sec, s, t): max logit, its lowest
+// id, second largest logit, s = sum e^(x-m), t = sum e^(x-m) (x-m); then
+// lse = m + log s and entropy = log s - t/s.
+#include <cuda.h>
+#include <math.h>
+
+#include "cospec_device.cuh"
+#include "cospec_internal.h"
+
+namespace cospec {
+
+namespace {
+
+constexpr int BM = 128;                 // vocab rows per tile (MMA M)
+constexpr int BK = 64;                  // K elements per stage (one 128-byte swizzle row)
+constexpr int A_BYTES = BM * BK * 2;    // 16 KB
+constexpr int NUM_THREADS = 192;        // TMA warp, MMA warp, 4 epilogue warps
+constexpr int EPI_THREADS = 128;
+constexpr int MAX_ROWS = 256;           // rows per pass
+constexpr uint64_t WAIT_NS = 2000000000ull;
+
+struct Stat {
+  float m;
+  int i;
+  float sec;
+  float s;
+  float t;
+};
+
+CS_DEV Stat stat_identity() { return Stat{-INFINITY, 0x7fffffff, -INFINITY, 0.f, 0.f}; }
+
+CS_DEV Stat stat_merge(const Stat& a, const Stat& b) {
+  const bool a_hi = (a.m > b.m) || (a.m == b.m && a.i < b.i);
+  const Stat& hi = a_hi ? a : b;
+  const Stat& lo = a_hi ? b : a;
+  Stat r;
+  r.m = hi.m;
+  r.i = hi.i;
+  r.sec = fmaxf(fmaxf(hi.sec, lo.sec), lo.m);
+  if (lo.s > 0.f) {
+    const float dm = lo.m - hi.m;
+    const float e = __expf(dm);
+    r.s = hi.s + lo.s * e;
+    r.t = hi.t + e * (lo.t + lo.s * dm);
+  } else {
+    r.s = hi.s;
+    r.t = hi.t;
+  }
+  return r;
+}
+
+CS_DEV Stat stat_shfl_xor(const Stat& a, int off) {
+  Stat r;
+  r.m = __shfl_xor_sync(0xffffffffu, a.m, off);
+  r.i = __shfl_xor_sync(0xffffffffu, a.i, off);
+  r.sec = __shfl_xor_sync(0xffffffffu, a.sec, off);
+  r.s = __shfl_xor_sync(0xffffffffu, a.s, off);
+  r.t = __shfl_xor_sync(0xffffffffu, a.t, off);
+  return r;
+}
+
+CS_DEV Stat stat_of(float x, int v) {
+  return Stat{x, v, -INFINITY, (x == -INFINITY) ? 0.f : 1.f, 0.f};
+}
+
+// Reduce 16 columns held by every lane of a warp (lane l holds vocab id
+// base + l) so that lanes 2c and 2c+1 end with column c reduced over all 32
+// lanes.  Each butterfly level exchanges half of the remaining columns, so a
+// column costs about one merge per lane instead of five.
+CS_DEV Stat warp_reduce16(const float (&x)[16], int lane, int vid) {
+  Stat a[8];
+  {
+    const bool up = (lane & 16) != 0;
+    const int pv = vid ^ 16;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      const float send = up ? x[c] : x[c + 8];
+      const float keep = up ? x[c + 8] : x[c];
+      const float recv = __shfl_xor_sync(0xffffffffu, send, 16);
+      a[c] = stat_merge(stat_of(keep, vid), stat_of(recv, pv));
+    }
+  }
+  Stat b4[4];
+  {
+    const bool up = (lane & 8) != 0;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const Stat send = up ? a[c] : a[c + 4];
+      const Stat keep = up ? a[c + 4] : a[c];
+      b4[c] = stat_merge(keep, stat_shfl_xor(send, 8));
+    }
+  }
+  Stat c2[2];
+  {
+    const bool up = (lane & 4) != 0;
+#pragma unroll
+    for (int c = 0; c < 2; ++c) {
+      const Stat send = up ? b4[c] : b4[c + 2];
+      const Stat keep = up ? b4[c + 2] : b4[c];
+      c2[c] = stat_merge(keep, stat_shfl_xor(send, 4));
+    }
+  }
+  Stat d1;
+  {
+    const bool up = (lane & 2) != 0;
+    const Stat send = up ? c2[0] : c2[1];
+    const Stat keep = up ? c2[1] : c2[0];
+    d1 = stat_merge(keep, stat_shfl_xor(send, 2));
+  }
+  return stat_merge(d1, stat_shfl_xor(d1, 1));
+}
+
+struct LmParams {
+  const int32_t* draft_for_row;  // [M]
+  float* stats;                  // [M][5]
+  float4* part;                  // [gridDim.x][n_rows]: (m, sec, s, t)
+  int* part_idx;                 // [gridDim.x][n_rows]
+  int row0, n_rows, n_mma;
+  int d, V, num_tiles, stages;
+  uint32_t tmem_cols;
+  int* err;
+};
+
+struct SmemLayout {
+  uint32_t a_off, b_off, bar_off, epi_off, total;
+};
+
+__host__ __device__ inline SmemLayout lm_layout(int stages, int n_mma) {
+  SmemLayout L;
+  L.a_off = 0;
+  L.b_off = (uint32_t)stages * A_BYTES;
+  L.bar_off = L.b_off + (uint32_t)stages * n_mma * 128;
+  const uint32_t bar_bytes = (uint32_t)(2 * stages + 5) * 8 + 16;
+  L.epi_off = (L.bar_off + bar_bytes + 15) / 16 * 16;
+  // epilogue: per-warp tuples [4][n_mma] (float4 + int), running [n_mma] (float4 + int), draft ids
+  const uint32_t epi = 4u * n_mma * 20u + (uint32_t)n_mma * 20u + (uint32_t)n_mma * 4u + 16u;
+  L.total = L.epi_off + epi;
+  return L;
+}
+
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    lmhead_kernel(const __grid_constant__ CUtensorMap tmap_w,
+                  const __grid_constant__ CUtensorMap tmap_h, const LmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  // TMA with 128B swizzle and the UMMA descriptors need 1024-byte alignment.
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const SmemLayout L = lm_layout(p.stages, p.n_mma);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.bar_off);
+  uint64_t* empty = full + p.stages;
+  uint64_t* tfull = empty + p.stages;    // [2]
+  uint64_t* tempty = tfull + 2;          // [2]
+  uint64_t* mma_done = tempty + 2;       // [1]
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(mma_done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+  float4* s_wt = reinterpret_cast<float4*>(smem + L.epi_off);      // [4][n_mma]
+  int* s_wti = reinterpret_cast<int*>(s_wt + 4 * p.n_mma);         // [4][n_mma]
+  float4* s_run = reinterpret_cast<float4*>(s_wti + 4 * p.n_mma);  // [n_mma]
+  int* s_runi = reinterpret_cast<int*>(s_run + p.n_mma);           // [n_mma]
+  int* s_draft = s_runi + p.n_mma;                                 // [n_mma]
+  volatile int* s_fail = reinterpret_cast<volatile int*>(s_draft + p.n_mma);  // [4]
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int kblocks = p.d / BK;
+  const uint32_t b_bytes = (uint32_t)p.n_mma * 128u;
+
+  if (tid == 0) {
+    for (int s = 0; s < p.stages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(&tfull[0], 1);
+    mbar_init(&tfull[1], 1);
+    mbar_init(&tempty[0], EPI_THREADS);
+    mbar_init(&tempty[1], EPI_THREADS);
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+    tma_prefetch_desc(&tmap_w);
+    tma_prefetch_desc(&tmap_h);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_holder, p.tmem_cols);
+    tmem_relinquish();
+  }
+  if (warp >= 2) {
+    for (int c = tid - 64; c < p.n_mma; c += EPI_THREADS) {
+      s_run[c] = make_float4(-INFINITY, -INFINITY, 0.f, 0.f);
+      s_runi[c] = 0x7fffffff;
+      s_draft[c] = (c < p.n_rows) ? p.draft_for_row[p.row0 + c] : -2;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+  const uint32_t idesc = idesc_bf16_f32(BM, p.n_mma);
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      const uint64_t pol_w = l2_policy_evict_first();
+      const uint64_t pol_h = l2_policy_evict_last();
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued_mask = 0, issued_parity = 0;   // last load per stage (stages <= 16)
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, WAIT_NS) || *abort_flag) {
+            ok = false;
+            break;
+          }
+          const uint32_t sa = smem_u32(smem + L.a_off + (uint32_t)stage * A_BYTES);
+          const uint32_t sb = smem_u32(smem + L.b_off + (uint32_t)stage * b_bytes);
+          mbar_arrive_expect_tx(&full[stage], (uint32_t)A_BYTES + b_bytes);
+          tma_load_2d(sa, &tmap_w, &full[stage], kb * BK, tile * BM, pol_w);
+          tma_load_2d(sb, &tmap_h, &full[stage], kb * BK, p.row0, pol_h);
+          issued_mask |= 1u << stage;
+          issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
+          if (++stage == p.stages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        set_err(p.err, ERR_TIMEOUT);
+        *abort_flag = 1;
+        // let every issued copy land before shared memory is released
+        for (int s = 0; s < p.stages; ++s)
+          if (issued_mask & (1u << s)) mbar_wait(&full[s], (issued_parity >> s) & 1u, WAIT_NS);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      int it = 0;
+      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x, ++it) {
+        const int acc = it & 1;
+        const uint32_t aph = (uint32_t)(it >> 1) & 1u;
+        if (!mbar_wait(&tempty[acc], aph ^ 1u, WAIT_NS) || *abort_flag) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * p.n_mma);
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&full[stage], phase, WAIT_NS) || *abort_flag) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + L.a_off + (uint32_t)stage * A_BYTES);
+          const uint32_t sb = smem_u32(smem + L.b_off + (uint32_t)stage * b_bytes);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            umma_bf16(d_tmem, smem_desc_sw128(sa + k * 32), smem_desc_sw128(sb + k * 32), idesc,
+                      (kb | k) != 0 ? 1u : 0u);
+          }
+          umma_commit(&empty[stage]);
+          if (++stage == p.stages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit(&tfull[acc]);
+      }
+      if (!ok) {
+        set_err(p.err, ERR_TIMEOUT);
+        *abort_flag = 1;
+      }
+      // every MMA issued by this thread completes before TMEM is released
+      umma_commit(mma_done);
+      mbar_wait(mma_done, 0, WAIT_NS);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;               // TMEM lane quarter this warp may access
+    const int etid = tid - 64;
+    const int nchunks = (p.n_rows + 15) / 16;
+    int it = 0;
+    for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x, ++it) {
+      const int acc = it & 1;
+      const uint32_t aph = (uint32_t)(it >> 1) & 1u;
+      // The four epilogue warps take the abort decision together (named
+      // barrier + shared flags) so none of them is left waiting at a barrier.
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(&tfull[acc], aph, WAIT_NS));
+      if (lane == 0) s_fail[q] = ok ? 0 : 1;
+      named_bar_sync(1, EPI_THREADS);
+      if (s_fail[0] | s_fail[1] | s_fail[2] | s_fail[3]) {
+        if (etid == 0) {
+          set_err(p.err, ERR_TIMEOUT);
+          *abort_flag = 1;
+        }
+        break;
+      }
+      tc_fence_after();
+      const int vid = tile * BM + q * 32 + lane;
+      const bool valid = vid < p.V;
+      const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * p.n_mma);
+      for (int ch = 0; ch < nchunks; ++ch) {
+        float x[16];
+        tmem_ld16(tbase + (uint32_t)(ch * 16), x);
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+          const int col = ch * 16 + c;   // < n_mma; s_draft holds -2 past n_rows
+          if (valid && s_draft[col] == vid) p.stats[(size_t)(p.row0 + col) * 5 + 4] = x[c];
+          if (!valid) x[c] = -INFINITY;
+        }
+        const Stat r = warp_reduce16(x, lane, vid);
+        const int col = ch * 16 + (lane >> 1);
+        if ((lane & 1) == 0 && col < p.n_rows) {
+          s_wt[q * p.n_mma + col] = make_float4(r.m, r.sec, r.s, r.t);
+          s_wti[q * p.n_mma + col] = r.i;
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&tempty[acc]);
+      named_bar_sync(1, EPI_THREADS);
+      for (int col = etid; col < p.n_rows; col += EPI_THREADS) {
+        const float4 rv = s_run[col];
+        Stat acc_s{rv.x, s_runi[col], rv.y, rv.z, rv.w};
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          const float4 v = s_wt[w * p.n_mma + col];
+          acc_s = stat_merge(acc_s, Stat{v.x, s_wti[w * p.n_mma + col], v.y, v.z, v.w});
+        }
+        s_run[col] = make_float4(acc_s.m, acc_s.sec, acc_s.s, acc_s.t);
+        s_runi[col] = acc_s.i;
+      }
+      named_bar_sync(1, EPI_THREADS);
+    }
+    for (int col = etid; col < p.n_rows; col += EPI_THREADS) {
+      p.part[(size_t)blockIdx.x * p.n_rows + col] = s_run[col];
+      p.part_idx[(size_t)blockIdx.x * p.n_rows + col] = s_runi[col];
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc(tmem_base, p.tmem_cols);
+  }
+}
+
+// Merge the per-CTA partial statistics of every row (one warp per row).
+__global__ void __launch_bounds__(128) lmhead_reduce_kernel(const float4* part, const int* part_idx,
+                                                            int nparts, int row0, int n_rows,
+                                                            int V, const int32_t* draft_for_row,
+                                                            int32_t* argmax, float* stats, int* err) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row = blockIdx.x * 4 + warp;
+  if (row >= n_rows) return;
+  Stat a = stat_identity();
+  for (int c = lane; c < nparts; c += 32) {
+    const float4 v = part[(size_t)c * n_rows + row];
+    a = stat_merge(a, Stat{v.x, part_idx[(size_t)c * n_rows + row], v.y, v.z, v.w});
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) a = stat_merge(a, stat_shfl_xor(a, off));
+  if (lane == 0) {
+    const int m = row0 + row;
+    float* st = stats + (size_t)m * 5;
+    const float ls = logf(a.s);
+    argmax[m] = a.i;
+    st[0] = a.m;
+    st[1] = a.sec;
+    st[2] = a.m + ls;
+    st[3] = ls - a.t / a.s;
+    const int dft = draft_for_row[m];
+    if (dft == -1) {
+      st[4] = __int_as_float(0x7fc00000);
+    } else if (dft < -1 || dft >= V) {
+      st[4] = __int_as_float(0x7fc00000);
+      set_err(err, ERR_TOKEN);
+    }
+  }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  }
+  return fn;
+}
+
+// 2-D bf16 row-major [rows, cols] map with a {64, box_rows} box and 128B swizzle.
+bool make_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+  EncodeTiledFn enc = get_encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+LmheadPlan plan_lmhead(int M, int d, int V, int num_sms) {
+  LmheadPlan pl{};
+  const int rows = M < MAX_ROWS ? M : MAX_ROWS;
+  pl.n_mma = (rows + 15) / 16 * 16;
+  if (pl.n_mma < 16) pl.n_mma = 16;
+  pl.passes = (M + MAX_ROWS - 1) / MAX_ROWS;
+  pl.num_tiles = (V + BM - 1) / BM;
+  pl.grid = pl.num_tiles < num_sms ? pl.num_tiles : num_sms;
+  const uint32_t budget = 227u * 1024u - 1024u;
+  const uint32_t fixed = lm_layout(0, pl.n_mma).total;
+  const uint32_t per_stage = A_BYTES + (uint32_t)pl.n_mma * 128u;
+  int st = (int)((budget - fixed) / per_stage);
+  if (st > 12) st = 12;
+  pl.stages = st;
+  pl.smem_bytes = lm_layout(st, pl.n_mma).total + 1024;
+  const size_t per_part = (size_t)1024 * MAX_ROWS;  // upper bound on CTAs x rows
+  pl.ws_bytes = per_part * sizeof(float4) + per_part * sizeof(int);
+  return pl;
+}
+
+cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
+                          const __nv_bfloat16* w, const int32_t* draft_for_row, int32_t* argmax,
+                          float* stats, void* ws, const LmheadPlan& pl, int* err,
+                          cudaStream_t stream) {
+  CUtensorMap map_w, map_h;
+  if (!make_map(&map_w, w, (uint64_t)V, (uint64_t)d, BM)) return cudaErrorInvalidValue;
+  if (!make_map(&map_h, hidden, (uint64_t)M, (uint64_t)d, (uint32_t)pl.n_mma))
+    return cudaErrorInvalidValue;
+  static bool configured[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 64 && !configured[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(lmhead_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         227 * 1024);
+    if (e != cudaSuccess) return e;
+    configured[dev] = true;
+  }
+  float4* part = static_cast<float4*>(ws);
+  int* part_idx = reinterpret_cast<int*>(part + (size_t)1024 * MAX_ROWS);
+  uint32_t tmem_cols = 32;
+  while (tmem_cols < (uint32_t)(2 * pl.n_mma)) tmem_cols <<= 1;
+  for (int pass = 0; pass < pl.passes; ++pass) {
+    LmParams p{};
+    p.draft_for_row = draft_for_row;
+    p.stats = stats;
+    p.part = part;
+    p.part_idx = part_idx;
+    p.row0 = pass * MAX_ROWS;
+    p.n_rows = (M - p.row0) < MAX_ROWS ? (M - p.row0) : MAX_ROWS;
+    p.n_mma = pl.n_mma;
+    p.d = d;
+    p.V = V;
+    p.num_tiles = pl.num_tiles;
+    p.stages = pl.stages;
+    p.tmem_cols = tmem_cols;
+    p.err = err;
+    lmhead_kernel<<<pl.grid, NUM_THREADS, pl.smem_bytes, stream>>>(map_w, map_h, p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    lmhead_reduce_kernel<<<(p.n_rows + 3) / 4, 128, 0, stream>>>(
+        part, part_idx, pl.grid, p.row0, p.n_rows, V, draft_for_row, argmax, stats, err);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace cospec

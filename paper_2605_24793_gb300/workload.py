@@ -155,17 +155,39 @@ def page_table(cfg: RoundConfig, ctx: np.ndarray, extra_tokens: int = 0):
     return table, num_pages
 
 
+# Tensors up to this many elements are drawn with NumPy's PCG64 generator on
+# the host, so they are bit-identical on every machine; larger ones are drawn
+# on the target device by torch's generator (same seed, device-specific stream).
+HOST_DRAW_LIMIT = 1 << 25
+
+
 def _gen(cfg: RoundConfig, tensor: str, device) -> torch.Generator:
     g = torch.Generator(device=device)
     g.manual_seed(seed_of(cfg, tensor))
     return g
 
 
-def _randn_bf16(shape, std, g, device, out=None):
-    if out is None:
-        out = torch.empty(shape, dtype=torch.bfloat16, device=device)
-    out.normal_(0.0, std, generator=g)
-    return out
+class _Normal:
+    """N(0, std^2) bf16 draws for one named tensor of a config."""
+
+    def __init__(self, cfg: RoundConfig, tensor: str, total: int, device):
+        self.host = total <= HOST_DRAW_LIMIT
+        self.device = torch.device(device)
+        if self.host:
+            self.rng = np.random.default_rng(seed_of(cfg, tensor))
+        else:
+            self.g = _gen(cfg, tensor, self.device)
+
+    def fill(self, out: torch.Tensor, std: float) -> torch.Tensor:
+        if self.host:
+            v = self.rng.standard_normal(tuple(out.shape), dtype=np.float32) * np.float32(std)
+            out.copy_(torch.from_numpy(v).to(torch.bfloat16))
+        else:
+            out.normal_(0.0, std, generator=self.g)
+        return out
+
+    def new(self, shape, std: float) -> torch.Tensor:
+        return self.fill(torch.empty(shape, dtype=torch.bfloat16, device=self.device), std)
 
 
 def mlp_params(cfg: RoundConfig, hidden: Optional[int] = None):
@@ -200,18 +222,21 @@ def make_round_inputs(cfg: RoundConfig, device="cpu", extra_tokens: int = 0,
     table, num_pages = page_table(cfg, ctx, extra_tokens)
     out: Dict[str, object] = dict(cfg=cfg, ctx_len_np=ctx, page_table_np=table,
                                   num_pages=num_pages, alias_layers=alias_layers)
-    out["q"] = _randn_bf16((L, B, R, Hq, D), cfg.qkv_std, _gen(cfg, "q", device), device)
-    out["k_blk"] = _randn_bf16((L, B, R, Hkv, D), cfg.qkv_std, _gen(cfg, "k_blk", device), device)
-    out["v_blk"] = _randn_bf16((L, B, R, Hkv, D), cfg.qkv_std, _gen(cfg, "v_blk", device), device)
+    def draw(name, shape, std):
+        return _Normal(cfg, name, int(np.prod(shape)), device).new(shape, std)
+
+    out["q"] = draw("q", (L, B, R, Hq, D), cfg.qkv_std)
+    out["k_blk"] = draw("k_blk", (L, B, R, Hkv, D), cfg.qkv_std)
+    out["v_blk"] = draw("v_blk", (L, B, R, Hkv, D), cfg.qkv_std)
     Lp = 1 if alias_layers else L
     for name in ("k_pages", "v_pages"):
         pool = torch.empty((Lp, num_pages, Hkv, P, D), dtype=torch.bfloat16, device=device)
-        g = _gen(cfg, name, device)
+        src = _Normal(cfg, name, pool.numel(), device)
         for l in range(Lp):           # layer by layer keeps the temporary small
-            _randn_bf16(None, cfg.qkv_std, g, device, out=pool[l])
+            src.fill(pool[l], cfg.qkv_std)
         out[name] = pool
-    out["hidden"] = _randn_bf16((B * R, cfg.hidden), cfg.h_std, _gen(cfg, "hidden", device), device)
-    out["w"] = _randn_bf16((cfg.vocab, cfg.hidden), cfg.w_std, _gen(cfg, "w", device), device)
+    out["hidden"] = draw("hidden", (B * R, cfg.hidden), cfg.h_std)
+    out["w"] = draw("w", (cfg.vocab, cfg.hidden), cfg.w_std)
     out["mlp"] = mlp_params(cfg)
     out["page_table"] = torch.from_numpy(table).to(device)
     out["ctx_len"] = torch.from_numpy(ctx).to(device)

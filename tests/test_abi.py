@@ -1,0 +1,107 @@
+"""The C-ABI library builds for sm_103a, loads, exports every entry point of
+include/cospec.h, and rejects bad arguments on the host before launching
+anything (no GPU needed)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2605_24793_gb300 import build as B
+from paper_2605_24793_gb300 import cospec as C
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    path = B.build()
+    return C.load_library(path)
+
+
+def _header_functions():
+    text = open(os.path.join(ROOT, "include", "cospec.h")).read()
+    return sorted(set(re.findall(r"COSPEC_API\s+[\w\s\*]+?\b(cospec_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_four_round_calls():
+    names = _header_functions()
+    for n in ("cospec_verify_attn", "cospec_lmhead_argmax_features", "cospec_arbitrate",
+              "cospec_accept_commit"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    names = _header_functions()
+    assert len(names) >= 10
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(names) == set(C.EXPORTED)
+
+
+def test_status_strings(lib):
+    assert lib.cospec_status_string(0) == b"ok"
+    assert lib.cospec_status_string(-1) == b"invalid argument"
+    assert lib.cospec_status_string(-3) == b"workspace missing or too small"
+    assert lib.cospec_status_string(123) == b"unknown status"
+
+
+def _dims(**kw):
+    d = dict(batch=2, rows=6, num_q_heads=32, num_kv_heads=8, head_dim=128, page_size=16,
+             max_pages_per_seq=300, num_pages=600, softmax_scale=0.0)
+    d.update(kw)
+    return C.AttnDims(*d.values())
+
+
+def test_attention_host_validation(lib):
+    f = lib.cospec_verify_attn
+    nul = None
+    # null pointers are rejected before any CUDA call
+    assert f(ctypes.byref(_dims()), 4096, *([nul] * 8), nul, 0, nul) == -1
+    # shapes the kernels do not cover
+    assert f(ctypes.byref(_dims(head_dim=96)), 4096, *([nul] * 8), nul, 0, nul) == -2
+    assert f(ctypes.byref(_dims(page_size=32)), 4096, *([nul] * 8), nul, 0, nul) == -2
+    assert f(ctypes.byref(_dims(rows=33)), 4096, *([nul] * 8), nul, 0, nul) == -2
+    assert f(ctypes.byref(_dims(num_q_heads=30)), 4096, *([nul] * 8), nul, 0, nul) == -1
+    assert f(ctypes.byref(_dims(softmax_scale=float("nan"))), 4096, *([nul] * 8), nul, 0, nul) == -1
+    # max_ctx beyond the page-table row
+    assert f(ctypes.byref(_dims()), 300 * 16 + 1, *([nul] * 8), nul, 0, nul) == -1
+    # empty batch is a no-op
+    assert f(ctypes.byref(_dims(batch=0)), 0, *([nul] * 8), nul, 0, nul) == 0
+    assert lib.cospec_verify_attn_ticket_bytes(ctypes.byref(_dims(batch=3, num_kv_heads=8))) == 256
+
+
+def test_lmhead_host_validation(lib):
+    f = lib.cospec_lmhead_argmax_features
+    assert f(0, 4096, 1000, *([None] * 6), 0, None) == 0          # no rows: nothing to do
+    assert f(4, 4096, 1000, *([None] * 6), 0, None) == -1         # null pointers
+    assert f(-1, 4096, 1000, *([None] * 6), 0, None) == -1
+    fake = ctypes.c_void_p(1 << 20)                                # never dereferenced
+    assert f(4, 4000, 1000, fake, fake, fake, fake, fake, fake, 1 << 30, None) == -2   # d % 64
+    assert f(4, 4096, 1000, ctypes.c_void_p((1 << 20) + 2), fake, fake, fake, fake, fake,
+             1 << 30, None) == -1                                  # misaligned hidden
+    assert lib.cospec_lmhead_workspace(6, 4096, 151936) > 0
+
+
+def test_arbitrate_host_validation(lib):
+    f = lib.cospec_arbitrate
+    fake = ctypes.c_void_p(1 << 20)
+    assert f(4, 32, fake, fake, fake, 16, fake, fake, fake, 0.0, 0.6, 0, fake, fake, None) == -2
+    assert f(4, 5, fake, fake, fake, 16, fake, fake, fake, 0.0, 0.6, 3, fake, fake, None) == -1
+    assert f(4, 5, fake, fake, fake, 16, fake, fake, fake, 0.0, float("nan"), 0, fake, fake, None) == -1
+    assert f(4, 5, fake, fake, fake, 16, None, fake, fake, 0.0, 0.6, 0, fake, fake, None) == -1
+    assert f(4, 5, fake, fake, fake, 2048, fake, fake, fake, 0.0, 0.6, 0, fake, fake, None) == -2
+    assert f(0, 5, None, None, None, 16, None, None, None, 0.0, 0.6, 0, None, None, None) == 0
+
+
+def test_commit_host_validation(lib):
+    f = lib.cospec_accept_commit
+    fake = ctypes.c_void_p(1 << 20)
+    d = _dims(batch=2, rows=6)
+    args = [fake] * 7
+    # batch in dims must match B, rows must be K + 1
+    assert f(3, 5, 36, ctypes.byref(d), *args, 10 ** 9, fake, fake, fake, fake, None) == -1
+    assert f(2, 4, 36, ctypes.byref(d), *args, 10 ** 9, fake, fake, fake, fake, None) == -1
+    # layer stride smaller than one pool
+    assert f(2, 5, 36, ctypes.byref(d), *args, 1024, fake, fake, fake, fake, None) == -1
+    assert f(2, 5, 36, ctypes.byref(d), *([None] * 7), 10 ** 9, fake, fake, fake, fake, None) == -1

@@ -1,0 +1,355 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle on seeded
+inputs small enough for the oracle, spanning several tiles, ragged tails and
+the degenerate cases (empty context, K = 0, single / many KV splits)."""
+import ctypes
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import cospec_oracle as O
+from paper_2605_24793_gb300 import build as BLD
+from paper_2605_24793_gb300 import cospec as C
+from paper_2605_24793_gb300 import workload as W
+from paper_2605_24793_gb300.round import VerifyRound
+
+from .parity_util import assert_close, tie_affected
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    C.load_library(BLD.build())
+    torch.cuda.set_device(0)
+    assert C.get_device_error() == 0
+    yield
+    assert C.get_device_error() == 0
+
+
+def bf16(a: np.ndarray) -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(torch.bfloat16).cuda()
+
+
+def host(t: torch.Tensor) -> np.ndarray:
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def _paged_case(rng, B, R, Hq, Hkv, D, ctx, shuffled, std=1.0, spare_pages=0):
+    P = 16
+    need = [(c + R + P - 1) // P for c in ctx]
+    num = sum(need) + spare_pages
+    order = rng.permutation(num) if shuffled else np.arange(num)
+    table = np.full((B, max(need)), -1, dtype=np.int32)
+    s = 0
+    for b in range(B):
+        table[b, :need[b]] = order[s:s + need[b]]
+        s += need[b]
+    mk = lambda *shape: rng.standard_normal(shape).astype(np.float32) * std
+    return dict(q=bf16(mk(B, R, Hq, D)), k_blk=bf16(mk(B, R, Hkv, D)), v_blk=bf16(mk(B, R, Hkv, D)),
+                k_pages=bf16(mk(num, Hkv, P, D)), v_pages=bf16(mk(num, Hkv, P, D)),
+                page_table=torch.from_numpy(table).cuda(),
+                ctx_len=torch.tensor(ctx, dtype=torch.int32).cuda(), table_np=table,
+                ctx_np=np.array(ctx))
+
+
+ATTN_CASES = [
+    # B, R, Hq, Hkv, D, contexts, shuffled pages
+    (1, 6, 32, 8, 128, [4096], False),              # Qwen3-8B-like, many KV splits
+    (4, 8, 64, 8, 128, [0, 17, 1000, 3333], True),  # G*R = 64 rows, empty and ragged contexts
+    (1, 5, 8, 2, 64, [256], False),                 # head_dim 64
+    (3, 3, 4, 4, 128, [5, 64, 65], True),           # G = 1, R = 3 -> 3 rows (one 16-row tile)
+    (2, 16, 64, 8, 128, [100, 2000], True),         # G*R = 128 rows (8 warps)
+    (2, 8, 128, 8, 64, [31, 700], False),           # G = 16 -> 128 rows at head_dim 64
+    (2, 1, 32, 8, 128, [0, 1], False),              # K = 0: one row per sequence
+    (5, 4, 32, 8, 128, [8191, 40, 63, 64, 2049], True),
+]
+
+
+@pytest.mark.parametrize("case", ATTN_CASES, ids=lambda c: f"B{c[0]}R{c[1]}G{c[2]//c[3]}D{c[4]}")
+def test_verify_attention_matches_oracle(case):
+    B, R, Hq, Hkv, D, ctx, shuffled = case
+    rng = np.random.default_rng(B * 1000 + R * 100 + Hq + D + sum(ctx))
+    t = _paged_case(rng, B, R, Hq, Hkv, D, ctx, shuffled)
+    max_ctx = max(ctx)
+    dims = C.attn_dims(t["q"], t["k_pages"], t["page_table"])
+    ws = C.new_attn_workspace(dims, max_ctx)
+    out = torch.empty_like(t["q"])
+    C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
+                  t["ctx_len"], out, ws, max_ctx)
+    ref = O.verify_attention(host(t["q"]), host(t["k_blk"]), host(t["v_blk"]), host(t["k_pages"]),
+                             host(t["v_pages"]), t["table_np"], t["ctx_np"], 16)
+    assert_close(host(out), ref, "attention")
+    # a second call on the same workspace (split counters must have been reset)
+    out2 = torch.empty_like(out)
+    C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
+                  t["ctx_len"], out2, ws, max_ctx)
+    assert torch.equal(out, out2)
+    nt = C.load_library().cospec_verify_attn_ticket_bytes(ctypes.byref(dims))
+    assert int(ws[:nt].sum()) == 0
+
+
+def test_verify_attention_split_count_does_not_change_result_beyond_tolerance():
+    rng = np.random.default_rng(3)
+    t = _paged_case(rng, 2, 6, 32, 8, 128, [3000, 5000], True)
+    ref = O.verify_attention(host(t["q"]), host(t["k_blk"]), host(t["v_blk"]), host(t["k_pages"]),
+                             host(t["v_pages"]), t["table_np"], t["ctx_np"], 16)
+    for max_ctx in (5000, t["table_np"].shape[1] * 16):     # different split plans
+        dims = C.attn_dims(t["q"], t["k_pages"], t["page_table"])
+        ws = C.new_attn_workspace(dims, max_ctx)
+        out = torch.empty_like(t["q"])
+        C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
+                      t["ctx_len"], out, ws, max_ctx)
+        assert_close(host(out), ref, f"attention max_ctx={max_ctx}")
+
+
+def test_verify_attention_constant_values():
+    # closed form: constant V gives that constant whatever the scores
+    rng = np.random.default_rng(4)
+    t = _paged_case(rng, 2, 6, 32, 8, 128, [777, 3], True)
+    t["v_pages"].fill_(0.375)
+    t["v_blk"].fill_(0.375)
+    dims = C.attn_dims(t["q"], t["k_pages"], t["page_table"])
+    ws = C.new_attn_workspace(dims, 777)
+    out = torch.empty_like(t["q"])
+    C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
+                  t["ctx_len"], out, ws, 777)
+    assert torch.all(out.float() == 0.375)
+
+
+LM_CASES = [
+    # M, d, V, weight std
+    (1, 64, 128, 0.1),
+    (5, 512, 4096, 0.02),
+    (6, 4096, 151936, 0.02),      # Qwen3-8B LM head, batch 1, K = 5
+    (17, 256, 1000, 0.1),         # vocabulary not a multiple of the 128-row tile
+    (128, 1024, 3000, 0.05),
+    (300, 128, 2048, 0.1),        # two 256-row passes
+    (256, 5120, 1280, 0.02),
+]
+
+
+@pytest.mark.parametrize("case", LM_CASES, ids=lambda c: f"M{c[0]}d{c[1]}V{c[2]}")
+def test_lmhead_matches_oracle(case):
+    M, d, V, wstd = case
+    rng = np.random.default_rng(M * 7 + d + V)
+    hidden = bf16(rng.standard_normal((M, d)))
+    w = bf16(rng.standard_normal((V, d)) * wstd)
+    dfr = rng.integers(0, V, M).astype(np.int32)
+    dfr[::3] = -1
+    dfr_t = torch.from_numpy(dfr).cuda()
+    am = torch.empty(M, dtype=torch.int32, device="cuda")
+    st = torch.empty((M, 5), dtype=torch.float32, device="cuda")
+    ws = C.new_lmhead_workspace(M, d, V)
+    C.lmhead_argmax_features(hidden, w, dfr_t, am, st, ws)
+    ref_am, ref_st = O.lmhead_stats(host(hidden), host(w), dfr)
+    assert_close(st.cpu().numpy(), ref_st, "lm-head stats")
+    margin = ref_st[:, 0] - ref_st[:, 1]
+    clear = margin >= 1e-3
+    assert np.array_equal(am.cpu().numpy()[clear], ref_am[clear])
+    print(f"lm-head {case}: tie rows {(~clear).sum()}")
+
+
+def test_lmhead_exact_ties_pick_lowest_id():
+    rng = np.random.default_rng(11)
+    M, d, V = 8, 256, 700
+    hidden = rng.standard_normal((M, d))
+    w = rng.standard_normal((V, d)) * 0.01
+    w[[3, 130, 699]] = hidden[0] * 0.5          # three identical top rows for row 0
+    w[[257, 258]] = hidden[1] * 0.5             # two identical top rows for row 1
+    hidden_t, w_t = bf16(hidden), bf16(w)
+    am = torch.empty(M, dtype=torch.int32, device="cuda")
+    st = torch.empty((M, 5), dtype=torch.float32, device="cuda")
+    C.lmhead_argmax_features(hidden_t, w_t, torch.full((M,), -1, dtype=torch.int32, device="cuda"),
+                             am, st, C.new_lmhead_workspace(M, d, V))
+    am = am.cpu().numpy()
+    st = st.cpu().numpy()
+    assert am[0] == 3 and am[1] == 257
+    assert st[0, 0] == st[0, 1] and st[1, 0] == st[1, 1]      # second == max on a tie
+    assert np.all(np.isnan(st[:, 4]))
+
+
+def _stats_case(rng, B, K, V=64):
+    x = rng.standard_normal((B * (K + 1), V)) * 2.0
+    top1 = np.argmax(x, axis=1).reshape(B, K + 1)
+    draft = np.where(rng.random((B, K)) < 0.5, top1[:, :K], rng.integers(0, V, (B, K))).astype(np.int32)
+    dfr = np.full((B, K + 1), -1)
+    dfr[:, :K] = draft
+    am, st = O.row_stats(x, dfr.reshape(-1))
+    return draft, am.reshape(B, K + 1).astype(np.int32), st.reshape(B, K + 1, 5)
+
+
+@pytest.mark.parametrize("K", [1, 3, 7, 31])
+@pytest.mark.parametrize("mode", [0, 1, 2])
+@pytest.mark.parametrize("lam", [0.4, 0.6, 0.8])
+def test_arbitrate_matches_oracle(K, mode, lam):
+    rng = np.random.default_rng(K * 100 + mode * 10 + int(lam * 10))
+    B, H = 37, 256
+    draft, am, st = _stats_case(rng, B, K)
+    w1 = (rng.random((H, 8)) * 2 - 1) / math.sqrt(8)
+    b1 = (rng.random(H) * 2 - 1) / math.sqrt(8)
+    w2 = (rng.random(H) * 2 - 1) / math.sqrt(H)
+    b2 = 0.05
+    ref_p, ref_a = O.arbitrate(draft, am, st, w1, b1, w2, b2, lam, mode)
+    p = torch.empty((B, K), dtype=torch.float32, device="cuda")
+    a = torch.empty((B, K), dtype=torch.uint8, device="cuda")
+    f32 = lambda v: torch.tensor(np.asarray(v, dtype=np.float32)).cuda()
+    C.arbitrate(torch.from_numpy(draft).cuda(), torch.from_numpy(am).cuda(),
+                f32(st), f32(w1), f32(b1), f32(w2), b2, lam, mode, p, a)
+    p = p.cpu().numpy()
+    a = a.cpu().numpy()
+    assert_close(p, ref_p, "policy probability")
+    clear = np.abs(ref_p - lam) >= 1e-3
+    assert np.array_equal(a[clear], ref_a[clear])
+    assert np.all(a[draft == am[:, :K]] == 1)
+
+
+def test_features_feed_the_mlp_as_the_oracle_builds_them():
+    # a one-hot first layer exposes each feature in turn through z
+    rng = np.random.default_rng(21)
+    B, K = 9, 7
+    draft, am, st = _stats_case(rng, B, K)
+    feats = O.arbitration_features(draft, am, st)
+    mism = draft != am[:, :K]
+    for k in range(8):
+        w1 = np.zeros((2, 8)); w1[0, k] = 1.0; w1[1, k] = -1.0
+        b1 = np.zeros(2); w2 = np.array([1.0, -1.0])           # z = relu(f) - relu(-f) = f_k
+        p = torch.empty((B, K), dtype=torch.float32, device="cuda")
+        a = torch.empty((B, K), dtype=torch.uint8, device="cuda")
+        f32 = lambda v: torch.tensor(np.asarray(v, dtype=np.float32)).cuda()
+        C.arbitrate(torch.from_numpy(draft).cuda(), torch.from_numpy(am).cuda(), f32(st), f32(w1),
+                    f32(b1), f32(w2), 0.0, 0.5, 0, p, a)
+        z = -np.log(1.0 / np.clip(p.cpu().numpy().astype(np.float64), 1e-30, 1 - 1e-7) - 1.0)
+        assert_close(z[mism], feats[..., k][mism], f"feature F{k}", abs_tol=1e-3, rel_tol=1e-3)
+
+
+@pytest.mark.parametrize("K", [0, 1, 5, 7])
+def test_accept_commit_matches_oracle(K):
+    rng = np.random.default_rng(40 + K)
+    L, B, R, Hkv, D, P = 3, 6, K + 1, 8, 128, 16
+    ctx = rng.integers(0, 200, B).astype(np.int32)
+    need = (ctx + R + P - 1) // P
+    num = int(need.sum())
+    perm = rng.permutation(num)
+    table = np.full((B, need.max()), -1, dtype=np.int32)
+    s0 = 0
+    for b in range(B):
+        table[b, :need[b]] = perm[s0:s0 + need[b]]
+        s0 += need[b]
+    V = 50
+    am = rng.integers(0, V, (B, R)).astype(np.int32)
+    draft = np.where(rng.random((B, K)) < 0.6, am[:, :K], rng.integers(0, V, (B, K))).astype(np.int32)
+    acc = (rng.random((B, K)) < 0.5).astype(np.uint8)
+    acc[draft == am[:, :K]] = 1
+    kb = bf16(rng.standard_normal((L, B, R, Hkv, D)))
+    vb = bf16(rng.standard_normal((L, B, R, Hkv, D)))
+    kp = bf16(rng.standard_normal((L, num, Hkv, P, D)))
+    vp = bf16(rng.standard_normal((L, num, Hkv, P, D)))
+    bits = lambda t: t.cpu().view(torch.int16).numpy()
+    kp0, vp0 = bits(kp), bits(vp)
+    ctx_t = torch.from_numpy(ctx).cuda()
+    alen = torch.empty(B, dtype=torch.int32, device="cuda")
+    em = torch.empty((B, R), dtype=torch.int32, device="cuda")
+    C.accept_commit(torch.from_numpy(draft.reshape(B, K)).cuda(), torch.from_numpy(am).cuda(),
+                    torch.from_numpy(acc.reshape(B, K)).cuda(), kb, vb, kp, vp,
+                    torch.from_numpy(table).cuda(), ctx_t, alen, em)
+    s, emitted = O.accept_scan(draft.reshape(B, K), am, acc.reshape(B, K))
+    kp_ref, vp_ref, ctx_ref = O.commit_kv(bits(kb), bits(vb), kp0, vp0, table, ctx, s, P)
+    assert np.array_equal(alen.cpu().numpy(), s)
+    assert np.array_equal(em.cpu().numpy(), emitted)
+    assert np.array_equal(ctx_t.cpu().numpy(), ctx_ref)
+    assert np.array_equal(bits(kp), kp_ref) and np.array_equal(bits(vp), vp_ref)
+
+
+def _tiny_round(mode, lam, cfg_name="tiny", **over):
+    cfg = W.CONFIGS[cfg_name].replace(**over) if over else W.CONFIGS[cfg_name]
+    inp = W.make_round_inputs(cfg, device="cuda")
+    hostinp = {k: (v.cpu() if torch.is_tensor(v) else v) for k, v in inp.items()}
+    x = O.lmhead_logits(hostinp["hidden"], hostinp["w"])
+    draft = W.synth_drafts(cfg, O.topk_ids(x, 8).reshape(cfg.batch, cfg.rows, 8))
+    ref = O.cospec_round(hostinp, draft, lam, mode)
+    rnd = VerifyRound(inp, draft, lam, mode, keep_attn=True)
+    rnd.run(restore=False)
+    torch.cuda.synchronize()
+    return cfg, draft, ref, rnd
+
+
+def _check_round(cfg, draft, ref, rnd, lam):
+    for l in range(cfg.layers):
+        assert_close(host(rnd.attn_out[l]), ref["attn"][l], f"attention layer {l}")
+    B, R, K = cfg.batch, cfg.rows, cfg.k
+    st = rnd.stats.cpu().numpy().reshape(B, R, 5)
+    assert_close(st, ref["stats"], "lm-head stats")
+    s_gpu = rnd.accept_len.cpu().numpy()
+    tie = tie_affected(ref["stats"], draft, ref["argmax"], ref["p"], ref["s"], s_gpu, lam)
+    ok = ~tie
+    am = rnd.argmax.cpu().numpy().reshape(B, R)
+    assert np.array_equal(am[ok], ref["argmax"][ok])
+    if K > 0:
+        assert_close(rnd.p.cpu().numpy()[ok], ref["p"][ok], "policy probability")
+        assert np.array_equal(rnd.accept.cpu().numpy()[ok], ref["a"][ok])
+    assert np.array_equal(s_gpu[ok], ref["s"][ok])
+    assert np.array_equal(rnd.emitted.cpu().numpy()[ok], ref["emitted"][ok])
+    assert np.array_equal(rnd.ctx_len.cpu().numpy()[ok], ref["ctx_len"][ok])
+    kp = rnd.k_pages.cpu().view(torch.int16).numpy()
+    vp = rnd.v_pages.cpu().view(torch.int16).numpy()
+    table = rnd.inp["page_table_np"]
+    for b in np.nonzero(ok)[0]:
+        pages = table[b][table[b] >= 0]
+        assert np.array_equal(kp[:, pages], ref["k_pages"][:, pages])
+        assert np.array_equal(vp[:, pages], ref["v_pages"][:, pages])
+    return int(tie.sum())
+
+
+@pytest.mark.parametrize("mode", [0, 1, 2])
+def test_tiny_round_matches_oracle(mode):
+    cfg, draft, ref, rnd = _tiny_round(mode, 0.6)
+    assert _check_round(cfg, draft, ref, rnd, 0.6) == 0
+    if mode == 1:
+        assert np.array_equal(ref["s"], O.strict_spd_length(draft, ref["argmax"]))
+    if mode == 2:
+        assert np.all(ref["s"] == cfg.k + 1)
+
+
+def test_small_batched_round_with_n01_inputs():
+    # several sequences, three layers, shuffled pages, N(0,1) attention inputs
+    cfg, draft, ref, rnd = _tiny_round(0, 0.6, batch=6, ctx_lo=0, ctx_hi=700, layers=3,
+                                       qkv_std=1.0, shuffled_pages=True, k=7, mismatch_rate=0.5)
+    ties = _check_round(cfg, draft, ref, rnd, 0.6)
+    print(f"tie-affected sequences: {ties} of {cfg.batch}")
+
+
+def test_block_size_one_round_is_greedy():
+    cfg, draft, ref, rnd = _tiny_round(0, 0.6, k=0, batch=3, ctx_lo=10, ctx_hi=300)
+    assert np.all(rnd.accept_len.cpu().numpy() == 1)
+    em = rnd.emitted.cpu().numpy()
+    x = O.lmhead_logits(rnd.hidden.cpu(), rnd.w.cpu())
+    assert np.array_equal(em[:, 0], np.argmax(x, axis=1))
+    _check_round(cfg, draft, ref, rnd, 0.6)
+
+
+def test_device_checks_set_error_bits_without_faulting():
+    rng = np.random.default_rng(5)
+    t = _paged_case(rng, 2, 6, 32, 8, 128, [100, 200], False)
+    dims = C.attn_dims(t["q"], t["k_pages"], t["page_table"])
+    ws = C.new_attn_workspace(dims, 200)
+    out = torch.empty_like(t["q"])
+    bad = t["page_table"].clone()
+    bad[1, 3] = 10 ** 6                                    # page id outside the pool
+    C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], bad, t["ctx_len"],
+                  out, ws, 200)
+    assert C.get_device_error() & C.DEVERR_PAGE
+    long_ctx = torch.tensor([100, t["table_np"].shape[1] * 16 + 1], dtype=torch.int32, device="cuda")
+    C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
+                  long_ctx, out, ws, 200)
+    assert C.get_device_error() & C.DEVERR_CTX
+    assert int(ws[:256].sum()) == 0                        # counters untouched by skipped units
+    M, d, V = 4, 128, 256
+    C.lmhead_argmax_features(bf16(rng.standard_normal((M, d))), bf16(rng.standard_normal((V, d))),
+                             torch.tensor([0, V, -1, 5], dtype=torch.int32, device="cuda"),
+                             torch.empty(M, dtype=torch.int32, device="cuda"),
+                             torch.empty((M, 5), dtype=torch.float32, device="cuda"),
+                             C.new_lmhead_workspace(M, d, V))
+    assert C.get_device_error() == C.DEVERR_TOKEN
+    assert C.get_device_error() == 0                       # reading clears the word
