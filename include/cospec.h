@@ -97,11 +97,9 @@ COSPEC_API int cospec_num_sms(void);
  *    ctx_len  int32 [batch]
  *    out      bf16 [batch, rows, num_q_heads, head_dim] (may not alias inputs)
  *    max_ctx  an upper bound of ctx_len[*] (host-side; sizes the KV split)
- *    ws       device workspace of at least cospec_verify_attn_workspace()
- *             bytes.  Its first cospec_verify_attn_ticket_bytes() bytes are
- *             split counters that must be zero before the first call
- *             (cudaMemset once); every completed call leaves them zero.
- *             Calls that run concurrently need distinct workspaces.
+ *    No workspace: the KV range of a (sequence, KV head) is split over the
+ *    CTAs of one thread-block cluster, whose partial results merge in
+ *    distributed shared memory.
  *    Supported: head_dim in {64, 128}; page_size == 16; rows <= 32;
  *    num_q_heads % num_kv_heads == 0; (num_q_heads / num_kv_heads) * rows <= 128.
  * ------------------------------------------------------------------------ */
@@ -117,13 +115,11 @@ typedef struct {
   float softmax_scale;   /* <= 0 selects 1/sqrt(head_dim) */
 } cospec_attn_dims;
 
-COSPEC_API size_t cospec_verify_attn_workspace(const cospec_attn_dims* dims, int max_ctx);
-COSPEC_API size_t cospec_verify_attn_ticket_bytes(const cospec_attn_dims* dims);
 COSPEC_API int cospec_verify_attn(const cospec_attn_dims* dims, int max_ctx,
                                   const uint16_t* q, const uint16_t* k_blk, const uint16_t* v_blk,
                                   const uint16_t* k_pages, const uint16_t* v_pages,
                                   const int32_t* page_table, const int32_t* ctx_len,
-                                  uint16_t* out, void* ws, size_t ws_bytes, void* stream);
+                                  uint16_t* out, void* stream);
 
 /* ------------------------------------------------------------------------ */
 /* 2. LM head fused with argmax and log-prob statistics (Eq. 2 gives the

@@ -20,7 +20,6 @@ POLICY_MLP, POLICY_TARGET, POLICY_DRAFT = 0, 1, 2
 DEVERR_PAGE, DEVERR_CTX, DEVERR_TOKEN, DEVERR_TIMEOUT = 1, 2, 4, 8
 
 EXPORTED = ("cospec_status_string", "cospec_get_device_error", "cospec_num_sms",
-            "cospec_verify_attn_workspace", "cospec_verify_attn_ticket_bytes",
             "cospec_verify_attn", "cospec_lmhead_workspace", "cospec_lmhead_argmax_features",
             "cospec_arbitrate", "cospec_accept_commit")
 
@@ -54,9 +53,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "cospec_status_string": (ctypes.c_char_p, [_i]),
         "cospec_get_device_error": (_i, [ctypes.POINTER(_i), _vp]),
         "cospec_num_sms": (_i, []),
-        "cospec_verify_attn_workspace": (_sz, [_PDIMS, _i]),
-        "cospec_verify_attn_ticket_bytes": (_sz, [_PDIMS]),
-        "cospec_verify_attn": (_i, [_PDIMS, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+        "cospec_verify_attn": (_i, [_PDIMS, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
         "cospec_lmhead_workspace": (_sz, [_i, _i, _i]),
         "cospec_lmhead_argmax_features": (_i, [_i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
         "cospec_arbitrate": (_i, [_i, _i, _vp, _vp, _vp, _i, _vp, _vp, _vp, _f, _f, _i, _vp, _vp, _vp]),
@@ -112,19 +109,7 @@ def num_sms() -> int:
     return load_library().cospec_num_sms()
 
 
-def verify_attn_workspace_bytes(dims: AttnDims, max_ctx: int) -> int:
-    return load_library().cospec_verify_attn_workspace(ctypes.byref(dims), max_ctx)
-
-
-def new_attn_workspace(dims: AttnDims, max_ctx: int, device="cuda") -> torch.Tensor:
-    """Workspace for cospec_verify_attn, zeroed (its split counters must start at 0)."""
-    n = verify_attn_workspace_bytes(dims, max_ctx)
-    if n == 0:
-        raise CospecError("unsupported attention geometry")
-    return torch.zeros(n, dtype=torch.uint8, device=device)
-
-
-def verify_attn(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len, out, ws, max_ctx,
+def verify_attn(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len, out, max_ctx,
                 softmax_scale: float = 0.0, stream=None) -> torch.Tensor:
     """Verify attention of one layer (Sec. 3.1, Eq. 2).  See include/cospec.h."""
     for t, n in ((q, "q"), (k_blk, "k_blk"), (v_blk, "v_blk"), (k_pages, "k_pages"),
@@ -132,7 +117,6 @@ def verify_attn(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len, out, ws,
         _req(t, torch.bfloat16, n)
     _req(page_table, torch.int32, "page_table", 2)
     _req(ctx_len, torch.int32, "ctx_len", 1)
-    _req(ws, torch.uint8, "ws", 1)
     dims = attn_dims(q, k_pages, page_table, softmax_scale)
     if tuple(k_blk.shape) != (dims.batch, dims.rows, dims.num_kv_heads, dims.head_dim):
         raise ValueError("k_blk shape does not match q / pages")
@@ -140,8 +124,7 @@ def verify_attn(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len, out, ws,
         raise ValueError("out must have q's shape")
     _check(load_library().cospec_verify_attn(
         ctypes.byref(dims), int(max_ctx), _ptr(q), _ptr(k_blk), _ptr(v_blk), _ptr(k_pages),
-        _ptr(v_pages), _ptr(page_table), _ptr(ctx_len), _ptr(out), _ptr(ws), ws.numel(),
-        _stream(stream)))
+        _ptr(v_pages), _ptr(page_table), _ptr(ctx_len), _ptr(out), _stream(stream)))
     return out
 
 

@@ -1,5 +1,6 @@
 // C ABI of the verify/arbitrate round: host-side validation, workspace
 // sizing, the device error word and dispatch to the kernel launchers.
+#include <cuda.h>
 #include <math.h>
 #include <stdint.h>
 
@@ -44,6 +45,38 @@ int* device_error_word() {
     g_err_ptr[dev] = static_cast<int*>(p);
   }
   return g_err_ptr[dev];
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+bool encode_tensor_map_bf16(void* map, const void* base, int rank, const uint64_t* dims,
+                            const uint64_t* strides, const uint32_t* box) {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return false;
+    fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  }
+  cuuint64_t d[3];
+  cuuint64_t st[2];
+  cuuint32_t bx[3], es[3];
+  for (int i = 0; i < rank; ++i) {
+    d[i] = dims[i];
+    bx[i] = box[i];
+    es[i] = 1;
+    if (i > 0) st[i - 1] = strides[i - 1];
+  }
+  return fn(static_cast<CUtensorMap*>(map), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank,
+            const_cast<void*>(base), d, st, bx, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace cospec
@@ -103,24 +136,30 @@ static int check_attn_dims(const cospec_attn_dims* d) {
   return COSPEC_OK;
 }
 
-COSPEC_API size_t cospec_verify_attn_workspace(const cospec_attn_dims* d, int max_ctx) {
-  if (check_attn_dims(d) != COSPEC_OK || max_ctx < 0) return 0;
-  const int sms = device_num_sms();
-  const AttnPlan pl = plan_verify_attn(d->batch, d->rows, d->num_q_heads, d->num_kv_heads,
-                                       d->head_dim, max_ctx, sms > 0 ? sms : 148);
-  return pl.total_bytes;
-}
-
-COSPEC_API size_t cospec_verify_attn_ticket_bytes(const cospec_attn_dims* d) {
-  if (check_attn_dims(d) != COSPEC_OK) return 0;
-  return (((size_t)d->batch * d->num_kv_heads * sizeof(int)) + 255) / 256 * 256;
+// Largest schedulable cluster not above `S` for this variant (cached per device).
+static int schedulable_cluster(int D, const AttnPlan& pl, int Hkv, int B) {
+  static int cache[64][2][4][5];   // [dev][D==128][mt index][log2 S] : 0 unknown, 1 ok, -1 no
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const int di = D == 128 ? 1 : 0;
+  const int mi = pl.mt == 1 ? 0 : pl.mt == 2 ? 1 : pl.mt == 4 ? 2 : 3;
+  int S = pl.cluster;
+  while (S > 1) {
+    int ls = 0;
+    while ((1 << ls) < S) ++ls;
+    int& c = cache[dev < 64 ? dev : 63][di][mi][ls];
+    if (c == 0) c = attn_max_active_clusters(D, pl.mt, pl.wk, S, Hkv, B) > 0 ? 1 : -1;
+    if (c > 0) break;
+    S >>= 1;
+  }
+  return S;
 }
 
 COSPEC_API int cospec_verify_attn(const cospec_attn_dims* d, int max_ctx, const uint16_t* q,
                                   const uint16_t* k_blk, const uint16_t* v_blk,
                                   const uint16_t* k_pages, const uint16_t* v_pages,
                                   const int32_t* page_table, const int32_t* ctx_len, uint16_t* out,
-                                  void* ws, size_t ws_bytes, void* stream) {
+                                  void* stream) {
   const int st = check_attn_dims(d);
   if (st != COSPEC_OK) return st;
   CS_CHECK_ARG(max_ctx >= 0 && max_ctx <= d->max_pages_per_seq * d->page_size);
@@ -130,9 +169,9 @@ COSPEC_API int cospec_verify_attn(const cospec_attn_dims* d, int max_ctx, const 
                aligned16(v_pages) && aligned16(out));
   const int sms = device_num_sms();
   if (sms <= 0) return COSPEC_ERR_CUDA;
-  const AttnPlan pl = plan_verify_attn(d->batch, d->rows, d->num_q_heads, d->num_kv_heads,
-                                       d->head_dim, max_ctx, sms);
-  if (!ws || ws_bytes < pl.total_bytes || !aligned16(ws)) return COSPEC_ERR_WORKSPACE;
+  AttnPlan pl = plan_verify_attn(d->batch, d->rows, d->num_q_heads, d->num_kv_heads,
+                                 d->head_dim, max_ctx, sms);
+  pl.cluster = schedulable_cluster(d->head_dim, pl, d->num_kv_heads, d->batch);
   int* err = device_error_word();
   if (!err) return COSPEC_ERR_CUDA;
   AttnArgs a{};
@@ -154,8 +193,6 @@ COSPEC_API int cospec_verify_attn(const cospec_attn_dims* d, int max_ctx, const 
   a.num_pages = d->num_pages;
   a.scale = d->softmax_scale > 0.f ? d->softmax_scale : 1.0f / sqrtf((float)d->head_dim);
   a.max_ctx = max_ctx;
-  a.ws = ws;
-  a.ws_bytes = ws_bytes;
   return from_cuda(launch_verify_attn(a, pl, err, static_cast<cudaStream_t>(stream)));
 }
 

@@ -12,6 +12,12 @@ namespace cospec {
 int device_num_sms();
 int* device_error_word();  // device address of the error word of the current device
 
+// cuTensorMapEncodeTiled for a bf16 tensor (rank 2 or 3, innermost first),
+// 128-byte swizzle, zero fill out of bounds.  dims/box in elements, strides
+// in bytes for dimensions 1..rank-1.
+bool encode_tensor_map_bf16(void* map, const void* base, int rank, const uint64_t* dims,
+                            const uint64_t* strides, const uint32_t* box);
+
 // ---------------------------------------------------------------- attention
 struct AttnArgs {
   const __nv_bfloat16* q;
@@ -25,14 +31,15 @@ struct AttnArgs {
   int B, R, Hq, Hkv, D, P, max_pages, num_pages;
   float scale;
   int max_ctx;
-  void* ws;
-  size_t ws_bytes;
 };
 struct AttnPlan {
-  int mt, wk, tiles_per_split, max_splits, nrp;
-  size_t ticket_bytes, partial_bytes, ml_bytes, total_bytes;
+  int mt, wk, nrp;
+  int cluster;            // CTAs per (sequence, KV head): the KV split
+  int tiles_per_split, max_splits;
+  size_t total_bytes;     // workspace (none)
 };
 AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int num_sms);
+int attn_max_active_clusters(int D, int mt, int wk, int S, int Hkv, int B);
 cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& plan, int* err,
                                cudaStream_t stream);
 

@@ -1,15 +1,19 @@
 // Verify attention of the K+1 block rows over a paged bf16 KV cache
 // (teacher-forced verification pass, Sec. 3.1 Eq. 2 of the paper).
 //
-// One CTA owns (sequence b, KV head, KV split).  It loads each 64-token K/V
-// tile of its split once (cp.async, 16-byte chunks, 3-stage ring, XOR-swizzled
-// rows) and multiplies it against ALL query rows that read this KV head: the
-// G = Hq/Hkv heads of the group times the R block rows (row index j*G + g).
-// Q.K^T and P.V run on bf16 tensor cores (mma.m16n8k16, fp32 accumulate);
-// the softmax is online in base 2.  Warps split the rows (16 per warp) and,
-// when there are few rows, the keys of a tile; their partial (m, l, O) merge
-// in shared memory.  Splits of one (b, head) merge through a workspace: the
-// last CTA to finish (atomic ticket, no waiting) combines them.
+// One CTA owns (sequence b, KV head, KV split).  The KV range of a (b, head)
+// is split over the CTAs of one thread-block cluster; every CTA streams its
+// 64-token K/V tiles (4 pages) once with TMA tensor loads -- one thread
+// issues a 16-row x 128-byte box per page and half-row, 128B-swizzled, into
+// a 3-stage mbarrier ring -- and multiplies each tile against ALL query rows
+// that read this KV head (the G = Hq/Hkv heads of the group times the R block
+// rows, row index j*G + g).  Q.K^T and P.V run on bf16 tensor cores
+// (mma.m16n8k16, fp32 accumulation), the softmax is online in base 2.  The
+// block's own keys (causal inside the block) ride the same ring as a final
+// tile of the last CTA of the cluster.  Partial (max, sum, O) of the cluster
+// merge through distributed shared memory, each CTA finishing a slice of the
+// rows, so no workspace and no extra launch are needed.
+#include <cuda.h>
 #include <math.h>
 
 #include "cospec_device.cuh"
@@ -19,333 +23,404 @@ namespace cospec {
 
 namespace {
 
-constexpr int KT = 64;        // keys per tile (4 pages of 16)
-constexpr int NSTAGE = 3;     // cp.async ring depth
-constexpr int PAGE = 16;      // page size (fixed)
+constexpr int KT = 64;            // keys per cache tile (4 pages)
+constexpr int PAGE = 16;          // page size (fixed)
+constexpr int ROWB = 128;         // bytes of one swizzled smem row (64 bf16)
+constexpr int BOX_BYTES = PAGE * ROWB;  // one page x 64 columns
+constexpr int NSTAGE = 3;
 
 struct AttnParams {
   const __nv_bfloat16* q;
-  const __nv_bfloat16* k_blk;
-  const __nv_bfloat16* v_blk;
-  const __nv_bfloat16* k_pages;
-  const __nv_bfloat16* v_pages;
   const int32_t* page_table;
   const int32_t* ctx_len;
   __nv_bfloat16* out;
-  float* ws_o;     // [B*Hkv][max_splits][nrp][D] un-normalised partial outputs
-  float2* ws_ml;   // [B*Hkv][max_splits][nrp] (running max, running sum), log2 domain
-  int* tickets;    // [B*Hkv] arrival counters, left at zero
-  int B, R, Hq, Hkv, G, NR, nrp;
+  int B, R, Hq, Hkv, G, NR;
   int max_pages, num_pages;
-  int tiles_per_split, max_splits;
   float scale_log2;
   int* err;
 };
 
 template <int D, int MT, int WK>
-__global__ void __launch_bounds__(MT* WK * 32) verify_attn_kernel(const AttnParams p) {
-  constexpr int NWARPS = MT * WK;
-  constexpr int NT = NWARPS * 32;
-  constexpr int KW = KT / WK;          // keys of a tile handled by one warp
-  constexpr int CH = D / 8;            // 16-byte chunks per key row
-  constexpr int TILE = KT * D;         // elements per K (or V) tile
-  constexpr int NRP = MT * 16;         // padded query rows
+struct Layout {
+  static constexpr int H = D / 64;                 // 128-byte halves of a key row
+  static constexpr int HALF = KT * ROWB;           // 8 KB: one half of a 64-key tile
+  static constexpr int STAGE = 2 * H * HALF;       // K halves then V halves
+  static constexpr int NRP = MT * 16;
+  static constexpr int RED = (WK > 1) ? MT * WK * 16 * (D * 4 + 8) : 0;
+  static constexpr int PART_O = RED;               // [NRP][D] fp32
+  static constexpr int PART_ML = PART_O + NRP * D * 4;   // [NRP] (m, l)
+  static constexpr int PART_END = PART_ML + NRP * 8;
+  static constexpr int BAR = NSTAGE * STAGE;       // full[NSTAGE], empty[NSTAGE]
+  static constexpr int TOTAL = BAR + 2 * NSTAGE * 8;
+  static_assert(PART_END <= NSTAGE * STAGE, "partials must fit in the stage ring");
+};
+
+// Online-softmax update of one warp's 16 rows with NK keys held in shared
+// memory (K and V, 128B-swizzled rows of 64 bf16, halves `half_bytes`
+// apart).  Key k of the region sits at smem row key0 + k and has index
+// kidx0 + k for masking; row r sees key index <= lim_r.
+template <int D, int NK>
+CS_DEV void attend(uint32_t sk, uint32_t sv, uint32_t half_bytes, int key0, int kidx0,
+                   bool need_mask, int lim0, int lim1, float scale_log2,
+                   const uint32_t (&qf)[D / 16][4], float (&o)[D / 8][4], float& m0, float& m1,
+                   float& l0, float& l1, int lane) {
+  const int c4 = lane & 3;
+  float s[NK / 8][4];
+#pragma unroll
+  for (int nt = 0; nt < NK / 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+#pragma unroll
+  for (int kk = 0; kk < D / 16; kk += 2) {
+    const int ch = kk * 2 + (lane >> 3);            // 16-byte chunk of the key row
+#pragma unroll
+    for (int nt = 0; nt < NK / 8; ++nt) {
+      const int key = key0 + nt * 8 + (lane & 7);
+      const uint32_t addr = sk + (uint32_t)(ch >> 3) * half_bytes + (uint32_t)key * ROWB +
+                            (uint32_t)(((ch & 7) ^ (key & 7)) * 16);
+      uint32_t b0, b1, b2, b3;
+      ldsm_x4(addr, b0, b1, b2, b3);
+      mma_16816(s[nt], qf[kk], b0, b1);
+      mma_16816(s[nt], qf[kk + 1], b2, b3);
+    }
+  }
+  float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+  for (int nt = 0; nt < NK / 8; ++nt) {
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      const int kidx = kidx0 + nt * 8 + 2 * c4 + e;
+      float v0 = s[nt][e] * scale_log2;
+      float v1 = s[nt][2 + e] * scale_log2;
+      if (need_mask) {
+        if (kidx > lim0) v0 = -INFINITY;
+        if (kidx > lim1) v1 = -INFINITY;
+      }
+      s[nt][e] = v0;
+      s[nt][2 + e] = v1;
+      mx0 = fmaxf(mx0, v0);
+      mx1 = fmaxf(mx1, v1);
+    }
+  }
+  mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+  mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+  mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+  mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+  const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+  const float base0 = (mn0 == -INFINITY) ? 0.f : mn0;
+  const float base1 = (mn1 == -INFINITY) ? 0.f : mn1;
+  const float a0 = exp2f(m0 - base0), a1 = exp2f(m1 - base1);
+  m0 = mn0;
+  m1 = mn1;
+  l0 *= a0;
+  l1 *= a1;
+#pragma unroll
+  for (int i = 0; i < D / 8; ++i) {
+    o[i][0] *= a0;
+    o[i][1] *= a0;
+    o[i][2] *= a1;
+    o[i][3] *= a1;
+  }
+  uint32_t pf[NK / 16][4];
+#pragma unroll
+  for (int nt = 0; nt < NK / 8; ++nt) {
+    const float p0 = exp2f(s[nt][0] - base0), p1 = exp2f(s[nt][1] - base0);
+    const float p2 = exp2f(s[nt][2] - base1), p3 = exp2f(s[nt][3] - base1);
+    l0 += p0 + p1;
+    l1 += p2 + p3;
+    pf[nt / 2][(nt % 2) * 2 + 0] = pack_bf16(p0, p1);
+    pf[nt / 2][(nt % 2) * 2 + 1] = pack_bf16(p2, p3);
+  }
+#pragma unroll
+  for (int kk2 = 0; kk2 < NK / 16; ++kk2) {
+    const int key = key0 + kk2 * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+    for (int nd = 0; nd < D / 8; nd += 2) {
+      const int ch = nd + (lane >> 4);
+      const uint32_t addr = sv + (uint32_t)(ch >> 3) * half_bytes + (uint32_t)key * ROWB +
+                            (uint32_t)(((ch & 7) ^ (key & 7)) * 16);
+      uint32_t b0, b1, b2, b3;
+      ldsm_x4_t(addr, b0, b1, b2, b3);
+      mma_16816(o[nd], pf[kk2], b0, b1);
+      mma_16816(o[nd + 1], pf[kk2], b2, b3);
+    }
+  }
+}
+
+template <int D, int MT, int WK>
+__global__ void __launch_bounds__(MT* WK * 32 + 32)
+    verify_attn_kernel(const __grid_constant__ CUtensorMap map_kp,
+                       const __grid_constant__ CUtensorMap map_vp,
+                       const __grid_constant__ CUtensorMap map_kb,
+                       const __grid_constant__ CUtensorMap map_vb, const AttnParams p) {
+  using LY = Layout<D, MT, WK>;
+  constexpr int NWARPS = MT * WK;        // consumer warps; warp NWARPS issues the loads
+  constexpr int NTC = NWARPS * 32;
+  constexpr int NTT = NTC + 32;
+  constexpr int KW = KT / WK;            // cache keys of a tile handled by one warp
+  constexpr int H = LY::H;
+  constexpr int NRP = LY::NRP;
+  constexpr int SMAX = 16;
   static_assert(KW % 16 == 0, "keys per warp must be a multiple of 16");
 
-  extern __shared__ __align__(128) uint8_t smem_raw[];
-  __nv_bfloat16* sK = reinterpret_cast<__nv_bfloat16*>(smem_raw);
-  __nv_bfloat16* sV = sK + NSTAGE * TILE;
-  __shared__ int s_last;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + LY::BAR);
+  uint64_t* empty = full + NSTAGE;
 
-  const int split = blockIdx.x, kvh = blockIdx.y, b = blockIdx.z;
+  const int S = (int)cluster_nctarank();
+  const int rank = (int)cluster_ctarank();
+  const int kvh = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int wr = warp / WK, wk = warp % WK;
 
   const int C = p.ctx_len[b];
-  const int T = C + p.R;
-  const int ntiles = (T + KT - 1) / KT;
-  const int nsplit = (ntiles + p.tiles_per_split - 1) / p.tiles_per_split;
-  if (C < 0 || C > p.max_pages * PAGE || nsplit > p.max_splits) {
-    if (split == 0 && kvh == 0 && tid == 0) set_err(p.err, ERR_CTX);
-    return;
-  }
-  if (split >= nsplit) return;
-  const int t_begin = split * p.tiles_per_split;
-  const int t_end = min(ntiles, t_begin + p.tiles_per_split);
-  const int* ptab = p.page_table + (size_t)b * p.max_pages;
+  const bool bad = (C < 0) || (C > p.max_pages * PAGE);
+  if (bad && rank == 0 && kvh == 0 && tid == 0) set_err(p.err, ERR_CTX);
+  // No early exit: every CTA of the cluster takes part in the merge below.
+  const int nct = bad ? 0 : (C + KT - 1) / KT;               // cache tiles of this sequence
+  const int tps = (nct + S - 1) / S;
+  const int t_begin = min(nct, rank * tps);
+  const int n = min(nct, t_begin + tps) - t_begin;
+  const bool do_blk = !bad && rank == S - 1;
+  const int nv = n + (do_blk ? 1 : 0);                       // virtual tiles (block last)
+  const int npages = (C + PAGE - 1) / PAGE;
+  const int KBR = (p.R + 15) & ~15;                          // block keys padded to 16
 
-  auto load_tile = [&](int t, int st) {
-    const uint32_t sk = smem_u32(sK + st * TILE);
-    const uint32_t sv = smem_u32(sV + st * TILE);
-#pragma unroll 4
-    for (int c = tid; c < KT * CH; c += NT) {
-      const int key = c / CH, ch = c % CH;
-      const int pos = t * KT + key;
-      const __nv_bfloat16* gk = p.k_pages;
-      const __nv_bfloat16* gv = p.v_pages;
-      bool valid = false;
-      if (pos < C) {
-        const int page = __ldg(ptab + pos / PAGE);
-        if ((unsigned)page < (unsigned)p.num_pages) {
-          const size_t off =
-              (((size_t)page * p.Hkv + kvh) * PAGE + (pos % PAGE)) * D + (size_t)ch * 8;
-          gk += off;
-          gv += off;
-          valid = true;
-        } else if (ch == 0) {
-          set_err(p.err, ERR_PAGE);
-        }
-      } else if (pos < T) {
-        const size_t off = (((size_t)b * p.R + (pos - C)) * p.Hkv + kvh) * D + (size_t)ch * 8;
-        gk = p.k_blk + off;
-        gv = p.v_blk + off;
-        valid = true;
-      }
-      const uint32_t so = (uint32_t)(key * D + ((ch ^ (key & 7)) * 8)) * 2u;
-      cp_async16(sk + so, gk, valid);
-      cp_async16(sv + so, gv, valid);
+  if (tid == 0) {
+    for (int s2 = 0; s2 < NSTAGE; ++s2) {
+      mbar_init(&full[s2], 1);
+      mbar_init(&empty[s2], NWARPS);
     }
-  };
-
-  // Issue the first tiles before anything else so the loads overlap set-up.
-#pragma unroll
-  for (int s = 0; s < NSTAGE - 1; ++s) {
-    if (t_begin + s < t_end) load_tile(t_begin + s, s);
-    cp_async_commit();
+    fence_barrier_init();
   }
-
-  // Query fragments (A operand, 16 rows x D) of this warp's row tile.
-  const int g_row = lane >> 2, c4 = lane & 3;
-  const int r0 = wr * 16 + g_row, r1 = r0 + 8;
-  uint32_t qf[D / 16][4];
-  {
-    auto row_ptr = [&](int r) -> const __nv_bfloat16* {
-      if (r >= p.NR) return nullptr;
-      const int j = r / p.G, g = r % p.G;
-      return p.q + (((size_t)b * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D;
-    };
-    const __nv_bfloat16* q0 = row_ptr(r0);
-    const __nv_bfloat16* q1 = row_ptr(r1);
-#pragma unroll
-    for (int kk = 0; kk < D / 16; ++kk) {
-      const int col = kk * 16 + 2 * c4;
-      qf[kk][0] = q0 ? __ldg(reinterpret_cast<const uint32_t*>(q0 + col)) : 0u;
-      qf[kk][1] = q1 ? __ldg(reinterpret_cast<const uint32_t*>(q1 + col)) : 0u;
-      qf[kk][2] = q0 ? __ldg(reinterpret_cast<const uint32_t*>(q0 + col + 8)) : 0u;
-      qf[kk][3] = q1 ? __ldg(reinterpret_cast<const uint32_t*>(q1 + col + 8)) : 0u;
-    }
-  }
-  // Block row of this thread's two query rows; a row j sees positions <= C + j.
-  const int lim0 = C + min(r0 / p.G, p.R - 1);
-  const int lim1 = C + min(r1 / p.G, p.R - 1);
+  __syncthreads();
 
   float o[D / 8][4];
-#pragma unroll
-  for (int i = 0; i < D / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
   float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+  const int g_row = lane >> 2, c4 = lane & 3;
+  const int wr = warp / WK, wk = warp % WK;
+  const int r0 = wr * 16 + g_row, r1 = r0 + 8;
 
-  for (int t = t_begin, it = 0; t < t_end; ++t, ++it) {
-    cp_async_wait<NSTAGE - 2>();
-    __syncthreads();
-    {
-      const int tn = t + NSTAGE - 1;
-      if (tn < t_end) load_tile(tn, (it + NSTAGE - 1) % NSTAGE);
-      cp_async_commit();
+  if (warp == NWARPS) {
+    // ---------------------------------------------------------- producer warp
+    if (lane == 0) {
+      tma_prefetch_desc(&map_kp);
+      tma_prefetch_desc(&map_vp);
     }
-    const int st = it % NSTAGE;
-    const uint32_t sk = smem_u32(sK + st * TILE);
-    const uint32_t sv = smem_u32(sV + st * TILE);
-
-    // S = Q K^T over this warp's KW keys.
-    float s[KW / 8][4];
-#pragma unroll
-    for (int nt = 0; nt < KW / 8; ++nt) {
-      s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-      const int key = wk * KW + nt * 8 + (lane & 7);
-#pragma unroll
-      for (int kk = 0; kk < D / 16; kk += 2) {
-        const int ch = kk * 2 + (lane >> 3);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(sk + (uint32_t)(key * D + ((ch ^ (key & 7)) * 8)) * 2u, b0, b1, b2, b3);
-        mma_16816(s[nt], qf[kk], b0, b1);
-        mma_16816(s[nt], qf[kk + 1], b2, b3);
+    const uint64_t pol = l2_policy_evict_first();
+    const int* ptab = p.page_table + (size_t)b * p.max_pages + (size_t)t_begin * 4;
+    const int my_pages = min(n * 4, npages - t_begin * 4);   // page-table entries of this CTA
+    int pid = 0;
+    for (int vt = 0; vt < nv; ++vt) {
+      if ((vt & 7) == 0) {                 // 32 page ids = the next 8 tiles, one per lane
+        const int e = vt * 4 + lane;
+        pid = (e < my_pages) ? __ldg(ptab + e) : 0;
       }
-    }
-
-    // Scale, causal mask on block positions, online softmax (log2 domain).
-    const int kbase = t * KT + wk * KW;
-    const bool need_mask = (t * KT + KT) > C;
-    float mx0 = -INFINITY, mx1 = -INFINITY;
+      const int st = vt % NSTAGE;
+      if (vt >= NSTAGE && !mbar_wait(&empty[st], (uint32_t)((vt / NSTAGE) - 1) & 1u))
+        set_err(p.err, ERR_TIMEOUT);
+      uint8_t* kb = smem + st * LY::STAGE;
+      uint8_t* vb = kb + H * LY::HALF;
+      if (vt < n) {
+        const int np = min(4, npages - (t_begin + vt) * 4);
+        int page[4];
 #pragma unroll
-    for (int nt = 0; nt < KW / 8; ++nt) {
+        for (int pg = 0; pg < 4; ++pg) page[pg] = __shfl_sync(0xffffffffu, pid, (vt & 7) * 4 + pg);
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&full[st], (uint32_t)(np * H * 2 * BOX_BYTES));
+          for (int pg = 0; pg < np; ++pg) {
+            int pgid = page[pg];
+            if ((unsigned)pgid >= (unsigned)p.num_pages) {
+              set_err(p.err, ERR_PAGE);
+              pgid = 0;
+            }
+            const int y = (pgid * p.Hkv + kvh) * PAGE;
 #pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const int pos = kbase + nt * 8 + 2 * c4 + e;
-        float v0 = s[nt][e] * p.scale_log2;
-        float v1 = s[nt][2 + e] * p.scale_log2;
-        if (need_mask) {
-          if (pos > lim0) v0 = -INFINITY;
-          if (pos > lim1) v1 = -INFINITY;
+            for (int h = 0; h < H; ++h) {
+              tma_load_2d(smem_u32(kb + h * LY::HALF + pg * BOX_BYTES), &map_kp, &full[st], h * 64, y, pol);
+              tma_load_2d(smem_u32(vb + h * LY::HALF + pg * BOX_BYTES), &map_vp, &full[st], h * 64, y, pol);
+            }
+          }
         }
-        s[nt][e] = v0;
-        s[nt][2 + e] = v1;
-        mx0 = fmaxf(mx0, v0);
-        mx1 = fmaxf(mx1, v1);
+      } else if (lane == 0) {
+        mbar_arrive_expect_tx(&full[st], (uint32_t)(H * 2 * ROWB * p.R));
+#pragma unroll
+        for (int h = 0; h < H; ++h) {
+          tma_load_3d(smem_u32(kb + h * LY::HALF), &map_kb, &full[st], h * 64, kvh, b * p.R, pol);
+          tma_load_3d(smem_u32(vb + h * LY::HALF), &map_vb, &full[st], h * 64, kvh, b * p.R, pol);
+        }
+      }
+      __syncwarp();
+    }
+  } else {
+    // ---------------------------------------------------------- consumer warps
+    // Query fragments (A operand, 16 rows x D) of this warp's row tile.
+    uint32_t qf[D / 16][4];
+    {
+      auto row_ptr = [&](int r) -> const __nv_bfloat16* {
+        if (r >= p.NR) return nullptr;
+        const int j = r / p.G, g = r % p.G;
+        return p.q + (((size_t)b * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D;
+      };
+      const __nv_bfloat16* q0 = row_ptr(r0);
+      const __nv_bfloat16* q1 = row_ptr(r1);
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const int col = kk * 16 + 2 * c4;
+        qf[kk][0] = q0 ? __ldg(reinterpret_cast<const uint32_t*>(q0 + col)) : 0u;
+        qf[kk][1] = q1 ? __ldg(reinterpret_cast<const uint32_t*>(q1 + col)) : 0u;
+        qf[kk][2] = q0 ? __ldg(reinterpret_cast<const uint32_t*>(q0 + col + 8)) : 0u;
+        qf[kk][3] = q1 ? __ldg(reinterpret_cast<const uint32_t*>(q1 + col + 8)) : 0u;
       }
     }
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-    const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-    const float base0 = (mn0 == -INFINITY) ? 0.f : mn0;
-    const float base1 = (mn1 == -INFINITY) ? 0.f : mn1;
-    const float a0 = exp2f(m0 - base0), a1 = exp2f(m1 - base1);
-    m0 = mn0;
-    m1 = mn1;
-    l0 *= a0;
-    l1 *= a1;
+    const int j0 = min(r0 / p.G, p.R - 1), j1 = min(r1 / p.G, p.R - 1);
 #pragma unroll
-    for (int i = 0; i < D / 8; ++i) {
-      o[i][0] *= a0;
-      o[i][1] *= a0;
-      o[i][2] *= a1;
-      o[i][3] *= a1;
-    }
-    uint32_t pf[KW / 16][4];
-#pragma unroll
-    for (int nt = 0; nt < KW / 8; ++nt) {
-      const float p0 = exp2f(s[nt][0] - base0), p1 = exp2f(s[nt][1] - base0);
-      const float p2 = exp2f(s[nt][2] - base1), p3 = exp2f(s[nt][3] - base1);
-      l0 += p0 + p1;
-      l1 += p2 + p3;
-      pf[nt / 2][(nt % 2) * 2 + 0] = pack_bf16(p0, p1);
-      pf[nt / 2][(nt % 2) * 2 + 1] = pack_bf16(p2, p3);
-    }
+    for (int i = 0; i < D / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
 
-    // O += P V.
-#pragma unroll
-    for (int kk2 = 0; kk2 < KW / 16; ++kk2) {
-      const int key = wk * KW + kk2 * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-#pragma unroll
-      for (int nd = 0; nd < D / 8; nd += 2) {
-        const int ch = nd + (lane >> 4);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(sv + (uint32_t)(key * D + ((ch ^ (key & 7)) * 8)) * 2u, b0, b1, b2, b3);
-        mma_16816(o[nd], pf[kk2], b0, b1);
-        mma_16816(o[nd + 1], pf[kk2], b2, b3);
+    for (int it = 0; it < nv; ++it) {
+      const int st = it % NSTAGE;
+      if (!mbar_wait(&full[st], (uint32_t)(it / NSTAGE) & 1u)) set_err(p.err, ERR_TIMEOUT);
+      uint8_t* kb = smem + st * LY::STAGE;
+      uint8_t* vb = kb + H * LY::HALF;
+      const bool is_blk = (it == n);
+      // Rows past the valid keys of this tile may hold stale or unwritten
+      // bytes: zero their V rows so that 0-weight keys contribute exactly 0.
+      const int valid_rows = is_blk ? p.R : min(KT, C - (t_begin + it) * KT);
+      const int zero_to = is_blk ? KBR : KT;
+      if (valid_rows < zero_to) {
+        const int nz = (zero_to - valid_rows) * H * (ROWB / 16);
+        for (int e = tid; e < nz; e += NTC) {
+          const int row = valid_rows + e / (H * (ROWB / 16));
+          const int rem = e % (H * (ROWB / 16));
+          *reinterpret_cast<uint4*>(vb + (rem / (ROWB / 16)) * LY::HALF + row * ROWB +
+                                    (rem % (ROWB / 16)) * 16) = make_uint4(0u, 0u, 0u, 0u);
+        }
+        fence_proxy_async_smem();
+        named_bar_sync(1, NTC);
+      }
+      if (!is_blk) {
+        const int kidx0 = (t_begin + it) * KT + wk * KW;
+        attend<D, KW>(smem_u32(kb), smem_u32(vb), LY::HALF, wk * KW, kidx0, valid_rows < KT,
+                      C - 1, C - 1, p.scale_log2, qf, o, m0, m1, l0, l1, lane);
+      } else if (wk == 0) {
+        if (KBR == 16)
+          attend<D, 16>(smem_u32(kb), smem_u32(vb), LY::HALF, 0, 0, true, j0, j1, p.scale_log2,
+                        qf, o, m0, m1, l0, l1, lane);
+        else
+          attend<D, 32>(smem_u32(kb), smem_u32(vb), LY::HALF, 0, 0, true, j0, j1, p.scale_log2,
+                        qf, o, m0, m1, l0, l1, lane);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[st]);
+    }
+    // After a timed-out wait a copy may still be in flight: wait (bounded)
+    // for the last fill of every stage before the ring is reused.
+    if (tid == 0) {
+      for (int st = 0; st < NSTAGE && st < nv; ++st) {
+        const int last = st + ((nv - 1 - st) / NSTAGE) * NSTAGE;
+        mbar_wait(&full[st], (uint32_t)(last / NSTAGE) & 1u);
       }
     }
+    l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+    l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
   }
-  cp_async_wait<0>();
   __syncthreads();
 
-  // Row sums live spread over the 4 threads of a quad.
-  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
-  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
-  l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
-  l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-
-  // Merge the WK key groups of each row tile in shared memory.
-  float* red_o = reinterpret_cast<float*>(smem_raw);           // [NWARPS][16][D]
-  float2* red_ml = reinterpret_cast<float2*>(red_o + NWARPS * 16 * D);  // [NWARPS][16]
-  {
-    float* wo = red_o + warp * 16 * D;
+  // CTA partial: rows of every warp, key groups merged (stage ring reused).
+  float* part_o = reinterpret_cast<float*>(smem + LY::PART_O);
+  float2* part_ml = reinterpret_cast<float2*>(smem + LY::PART_ML);
+  if constexpr (WK == 1) {
+    if (warp < NWARPS) {
 #pragma unroll
-    for (int nd = 0; nd < D / 8; ++nd) {
-      const int col = nd * 8 + 2 * c4;
-      *reinterpret_cast<float2*>(wo + g_row * D + col) = make_float2(o[nd][0], o[nd][1]);
-      *reinterpret_cast<float2*>(wo + (g_row + 8) * D + col) = make_float2(o[nd][2], o[nd][3]);
+      for (int nd = 0; nd < D / 8; ++nd) {
+        const int col = nd * 8 + 2 * c4;
+        *reinterpret_cast<float2*>(part_o + r0 * D + col) = make_float2(o[nd][0], o[nd][1]);
+        *reinterpret_cast<float2*>(part_o + r1 * D + col) = make_float2(o[nd][2], o[nd][3]);
+      }
+      if (c4 == 0) {
+        part_ml[r0] = make_float2(m0, l0);
+        part_ml[r1] = make_float2(m1, l1);
+      }
     }
-    if (c4 == 0) {
-      red_ml[warp * 16 + g_row] = make_float2(m0, l0);
-      red_ml[warp * 16 + g_row + 8] = make_float2(m1, l1);
+  } else {
+    float* red_o = reinterpret_cast<float*>(smem);                        // [NWARPS][16][D]
+    float2* red_ml = reinterpret_cast<float2*>(red_o + NWARPS * 16 * D);  // [NWARPS][16]
+    if (warp < NWARPS) {
+      float* wo = red_o + warp * 16 * D;
+#pragma unroll
+      for (int nd = 0; nd < D / 8; ++nd) {
+        const int col = nd * 8 + 2 * c4;
+        *reinterpret_cast<float2*>(wo + g_row * D + col) = make_float2(o[nd][0], o[nd][1]);
+        *reinterpret_cast<float2*>(wo + (g_row + 8) * D + col) = make_float2(o[nd][2], o[nd][3]);
+      }
+      if (c4 == 0) {
+        red_ml[warp * 16 + g_row] = make_float2(m0, l0);
+        red_ml[warp * 16 + g_row + 8] = make_float2(m1, l1);
+      }
+    }
+    __syncthreads();
+    for (int e = tid; e < NRP * (D / 4); e += NTT) {
+      const int r = e / (D / 4), c = (e % (D / 4)) * 4;
+      const int rt = r / 16, ri = r % 16;
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < WK; ++w) M = fmaxf(M, red_ml[(rt * WK + w) * 16 + ri].x);
+      float L = 0.f;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (M != -INFINITY) {
+#pragma unroll
+        for (int w = 0; w < WK; ++w) {
+          const float2 ml = red_ml[(rt * WK + w) * 16 + ri];
+          const float sc = exp2f(ml.x - M);
+          L += ml.y * sc;
+          const float4 v = *reinterpret_cast<const float4*>(red_o + ((rt * WK + w) * 16 + ri) * D + c);
+          acc.x += v.x * sc;
+          acc.y += v.y * sc;
+          acc.z += v.z * sc;
+          acc.w += v.w * sc;
+        }
+      }
+      *reinterpret_cast<float4*>(part_o + r * D + c) = acc;
+      if (c == 0) part_ml[r] = make_float2(M, L);
     }
   }
-  __syncthreads();
 
-  const bool single = (nsplit == 1);
-  const size_t bh = (size_t)b * p.Hkv + kvh;
-  float* part_o = p.ws_o + (bh * p.max_splits + split) * (size_t)p.nrp * D;
-  float2* part_ml = p.ws_ml + (bh * p.max_splits + split) * (size_t)p.nrp;
-  for (int e = tid; e < NRP * (D / 4); e += NT) {
+  // Merge the S partials of the cluster; CTA `rank` finishes every S-th chunk.
+  // All remote loads of an element are issued before any is consumed.
+  cluster_sync();
+  const uint32_t po = smem_u32(part_o), pml = smem_u32(part_ml);
+  for (int e = rank * NTT + tid; e < p.NR * (D / 4); e += S * NTT) {
     const int r = e / (D / 4), c = (e % (D / 4)) * 4;
-    const int rt = r / 16, ri = r % 16;
+    float2 ml[SMAX];
+    float4 v[SMAX];
+#pragma unroll
+    for (int s2 = 0; s2 < SMAX; ++s2) {
+      if (s2 < S) {
+        ml[s2] = dsmem_ld_f2(dsmem_map(pml + r * 8, s2));
+        v[s2] = dsmem_ld_f4(dsmem_map(po + (uint32_t)(r * D + c) * 4, s2));
+      }
+    }
     float M = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < WK; ++w) M = fmaxf(M, red_ml[(rt * WK + w) * 16 + ri].x);
+    for (int s2 = 0; s2 < SMAX; ++s2)
+      if (s2 < S) M = fmaxf(M, ml[s2].x);
     float L = 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     if (M != -INFINITY) {
 #pragma unroll
-      for (int w = 0; w < WK; ++w) {
-        const float2 ml = red_ml[(rt * WK + w) * 16 + ri];
-        const float sc = exp2f(ml.x - M);
-        L += ml.y * sc;
-        const float4 v = *reinterpret_cast<const float4*>(red_o + ((rt * WK + w) * 16 + ri) * D + c);
-        acc.x += v.x * sc;
-        acc.y += v.y * sc;
-        acc.z += v.z * sc;
-        acc.w += v.w * sc;
+      for (int s2 = 0; s2 < SMAX; ++s2) {
+        if (s2 < S) {
+          const float sc = (ml[s2].x == -INFINITY) ? 0.f : exp2f(ml[s2].x - M);
+          L += ml[s2].y * sc;
+          acc.x += v[s2].x * sc;
+          acc.y += v[s2].y * sc;
+          acc.z += v[s2].z * sc;
+          acc.w += v[s2].w * sc;
+        }
       }
     }
-    if (single) {
-      if (r < p.NR) {
-        const float inv = 1.f / L;
-        const int j = r / p.G, g = r % p.G;
-        __nv_bfloat16* dst = p.out + (((size_t)b * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D + c;
-        uint2 pk;
-        pk.x = pack_bf16(acc.x * inv, acc.y * inv);
-        pk.y = pack_bf16(acc.z * inv, acc.w * inv);
-        *reinterpret_cast<uint2*>(dst) = pk;
-      }
-    } else {
-      *reinterpret_cast<float4*>(part_o + (size_t)r * D + c) = acc;
-      if (c == 0) part_ml[r] = make_float2(M, L);
-    }
-  }
-  if (single) return;
-
-  // Last arriving split of this (b, head) merges every split.
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) {
-    const int prev = atomicAdd(p.tickets + bh, 1);
-    s_last = (prev == nsplit - 1);
-  }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-
-  float* wsc = reinterpret_cast<float*>(smem_raw);      // [nsplit][NRP] weights
-  float* inv_l = wsc + nsplit * NRP;                    // [NRP]
-  const float* all_o = p.ws_o + bh * p.max_splits * (size_t)p.nrp * D;
-  const float2* all_ml = p.ws_ml + bh * p.max_splits * (size_t)p.nrp;
-  for (int r = tid; r < NRP; r += NT) {
-    float M = -INFINITY;
-    for (int s2 = 0; s2 < nsplit; ++s2) M = fmaxf(M, __ldcg(&all_ml[(size_t)s2 * p.nrp + r].x));
-    float L = 0.f;
-    for (int s2 = 0; s2 < nsplit; ++s2) {
-      const float2 ml = __ldcg(&all_ml[(size_t)s2 * p.nrp + r]);
-      const float sc = (ml.x == -INFINITY) ? 0.f : exp2f(ml.x - M);
-      wsc[s2 * NRP + r] = sc;
-      L += ml.y * sc;
-    }
-    inv_l[r] = (L > 0.f) ? 1.f / L : 0.f;
-  }
-  __syncthreads();
-  for (int e = tid; e < p.NR * (D / 4); e += NT) {
-    const int r = e / (D / 4), c = (e % (D / 4)) * 4;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int s2 = 0; s2 < nsplit; ++s2) {
-      const float sc = wsc[s2 * NRP + r];
-      const float4 v = __ldcg(reinterpret_cast<const float4*>(all_o + ((size_t)s2 * p.nrp + r) * D + c));
-      acc.x += v.x * sc;
-      acc.y += v.y * sc;
-      acc.z += v.z * sc;
-      acc.w += v.w * sc;
-    }
-    const float inv = inv_l[r];
+    const float inv = (L > 0.f) ? 1.f / L : 0.f;
     const int j = r / p.G, g = r % p.G;
     __nv_bfloat16* dst = p.out + (((size_t)b * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D + c;
     uint2 pk;
@@ -353,110 +428,140 @@ __global__ void __launch_bounds__(MT* WK * 32) verify_attn_kernel(const AttnPara
     pk.y = pack_bf16(acc.z * inv, acc.w * inv);
     *reinterpret_cast<uint2*>(dst) = pk;
   }
-  if (tid == 0) p.tickets[bh] = 0;
+  cluster_sync();   // peers may still read this CTA's partial until here
 }
 
 template <int D, int MT, int WK>
-size_t attn_smem_bytes(int max_splits) {
-  const size_t pipe = (size_t)2 * NSTAGE * KT * D * sizeof(__nv_bfloat16);
-  const size_t red = (size_t)MT * WK * 16 * D * sizeof(float) + (size_t)MT * WK * 16 * sizeof(float2);
-  const size_t comb = ((size_t)max_splits * MT * 16 + MT * 16) * sizeof(float);
-  size_t s = pipe;
-  if (red > s) s = red;
-  if (comb > s) s = comb;
-  return s;
-}
-
-template <int D, int MT, int WK>
-cudaError_t launch_t(const AttnParams& p, dim3 grid, cudaStream_t stream) {
-  const size_t smem = attn_smem_bytes<D, MT, WK>(p.max_splits);
+cudaError_t launch_t(const CUtensorMap* maps, const AttnParams& p, int S, int B, int Hkv,
+                     cudaStream_t stream) {
+  using LY = Layout<D, MT, WK>;
+  const size_t smem = LY::TOTAL + 1024;
   static bool configured[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
+  auto kern = verify_attn_kernel<D, MT, WK>;
   if (dev < 64 && !configured[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(verify_attn_kernel<D, MT, WK>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
-  verify_attn_kernel<D, MT, WK><<<grid, MT * WK * 32, smem, stream>>>(p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(S, Hkv, B);
+  cfg.blockDim = dim3(MT * WK * 32 + 32, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = S;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], maps[2], maps[3], p);
 }
+
+template <int D, int MT, int WK>
+int max_cluster_t(int S, int Hkv, int B) {
+  using LY = Layout<D, MT, WK>;
+  auto kern = verify_attn_kernel<D, MT, WK>;
+  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(LY::TOTAL + 1024));
+  cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(S, Hkv, B);
+  cfg.blockDim = dim3(MT * WK * 32 + 32, 1, 1);
+  cfg.dynamicSmemBytes = LY::TOTAL + 1024;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = S;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
+int variant_mt(int NR) {
+  if (NR <= 16) return 1;
+  if (NR <= 32) return 2;
+  if (NR <= 64) return 4;
+  return 8;
+}
+
+#define COSPEC_ATTN_VARIANTS(X) \
+  X(128, 1, 4) X(128, 2, 2) X(128, 4, 1) X(128, 8, 1) X(64, 1, 4) X(64, 2, 2) X(64, 4, 1) X(64, 8, 1)
 
 }  // namespace
 
 AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int num_sms) {
   AttnPlan pl{};
-  const int G = Hq / Hkv;
-  const int NR = G * R;
-  int mt = (NR + 15) / 16;
-  if (mt <= 1) mt = 1;
-  else if (mt <= 2) mt = 2;
-  else if (mt <= 4) mt = 4;
-  else mt = 8;
-  pl.mt = mt;
-  pl.wk = (mt >= 4) ? 1 : 4 / mt;
-  pl.nrp = mt * 16;
-  const int tiles_max = (max_ctx + R + KT - 1) / KT;
-  const long long work = (long long)B * Hkv * tiles_max;
-  const int ctas_per_sm = (D == 64) ? 4 : 2;
-  const long long target = (long long)num_sms * ctas_per_sm * 6;   // about six waves
-  int tps = (int)((work + target - 1) / target);
-  if (tps < 2) tps = 2;
-  const int max_split_cap = 96;
-  if ((tiles_max + tps - 1) / tps > max_split_cap) tps = (tiles_max + max_split_cap - 1) / max_split_cap;
-  pl.tiles_per_split = tps;
-  pl.max_splits = (tiles_max + tps - 1) / tps;
-  pl.ticket_bytes = (((size_t)B * Hkv * sizeof(int)) + 255) / 256 * 256;
-  pl.partial_bytes = pl.max_splits > 1
-                         ? (size_t)B * Hkv * pl.max_splits * pl.nrp * D * sizeof(float)
-                         : 0;
-  pl.ml_bytes = pl.max_splits > 1 ? (size_t)B * Hkv * pl.max_splits * pl.nrp * sizeof(float2) : 0;
-  pl.ml_bytes = (pl.ml_bytes + 255) / 256 * 256;
-  pl.total_bytes = pl.ticket_bytes + pl.partial_bytes + pl.ml_bytes;
+  const int NR = (Hq / Hkv) * R;
+  pl.mt = variant_mt(NR);
+  pl.wk = (pl.mt >= 4) ? 1 : 4 / pl.mt;
+  pl.nrp = pl.mt * 16;
+  // Split each (sequence, head) over a cluster of S CTAs: enough CTAs for
+  // about four per SM over the launch, at least 4 cache tiles per CTA.
+  const int tiles = (max_ctx + KT - 1) / KT;
+  const long long units = (long long)B * Hkv;
+  const long long want = (4LL * num_sms + units - 1) / (units > 0 ? units : 1);
+  int S = 1;
+  while (S < 16 && S < want && (S * 2) * 4 <= tiles) S *= 2;
+  pl.cluster = S;
+  pl.tiles_per_split = (tiles + S - 1) / S;
+  pl.max_splits = S;
+  pl.total_bytes = 0;
   return pl;
+}
+
+int attn_max_active_clusters(int D, int mt, int wk, int S, int Hkv, int B) {
+#define X(DD, MM, WW) \
+  if (D == DD && mt == MM && wk == WW) return max_cluster_t<DD, MM, WW>(S, Hkv, B);
+  COSPEC_ATTN_VARIANTS(X)
+#undef X
+  return 0;
 }
 
 cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& pl, int* err,
                                cudaStream_t stream) {
+  CUtensorMap maps[4];
+  const uint64_t pool_rows = (uint64_t)a.num_pages * a.Hkv * PAGE;
+  const uint64_t dp[2] = {(uint64_t)a.D, pool_rows};
+  const uint64_t sp[1] = {(uint64_t)a.D * 2};
+  const uint32_t bp[2] = {64, PAGE};
+  const uint64_t db[3] = {(uint64_t)a.D, (uint64_t)a.Hkv, (uint64_t)a.B * a.R};
+  const uint64_t sb[2] = {(uint64_t)a.D * 2, (uint64_t)a.Hkv * a.D * 2};
+  const uint32_t bb[3] = {64, 1, (uint32_t)a.R};
+  if (!encode_tensor_map_bf16(&maps[0], a.k_pages, 2, dp, sp, bp) ||
+      !encode_tensor_map_bf16(&maps[1], a.v_pages, 2, dp, sp, bp) ||
+      !encode_tensor_map_bf16(&maps[2], a.k_blk, 3, db, sb, bb) ||
+      !encode_tensor_map_bf16(&maps[3], a.v_blk, 3, db, sb, bb))
+    return cudaErrorInvalidValue;
   AttnParams p{};
   p.q = a.q;
-  p.k_blk = a.k_blk;
-  p.v_blk = a.v_blk;
-  p.k_pages = a.k_pages;
-  p.v_pages = a.v_pages;
   p.page_table = a.page_table;
   p.ctx_len = a.ctx_len;
   p.out = a.out;
-  uint8_t* ws = static_cast<uint8_t*>(a.ws);
-  p.tickets = reinterpret_cast<int*>(ws);
-  p.ws_ml = reinterpret_cast<float2*>(ws + pl.ticket_bytes);
-  p.ws_o = reinterpret_cast<float*>(ws + pl.ticket_bytes + pl.ml_bytes);
   p.B = a.B;
   p.R = a.R;
   p.Hq = a.Hq;
   p.Hkv = a.Hkv;
   p.G = a.Hq / a.Hkv;
   p.NR = p.G * a.R;
-  p.nrp = pl.nrp;
   p.max_pages = a.max_pages;
   p.num_pages = a.num_pages;
-  p.tiles_per_split = pl.tiles_per_split;
-  p.max_splits = pl.max_splits;
   p.scale_log2 = a.scale * 1.4426950408889634f;
   p.err = err;
-  dim3 grid(pl.max_splits, a.Hkv, a.B);
-#define COSPEC_ATTN_CASE(DD, MM, WW) \
-  if (a.D == DD && pl.mt == MM && pl.wk == WW) return launch_t<DD, MM, WW>(p, grid, stream);
-  COSPEC_ATTN_CASE(128, 1, 4)
-  COSPEC_ATTN_CASE(128, 2, 2)
-  COSPEC_ATTN_CASE(128, 4, 1)
-  COSPEC_ATTN_CASE(128, 8, 1)
-  COSPEC_ATTN_CASE(64, 1, 4)
-  COSPEC_ATTN_CASE(64, 2, 2)
-  COSPEC_ATTN_CASE(64, 4, 1)
-  COSPEC_ATTN_CASE(64, 8, 1)
-#undef COSPEC_ATTN_CASE
+#define X(DD, MM, WW)                                      \
+  if (a.D == DD && pl.mt == MM && pl.wk == WW)             \
+    return launch_t<DD, MM, WW>(maps, p, pl.cluster, a.B, a.Hkv, stream);
+  COSPEC_ATTN_VARIANTS(X)
+#undef X
   return cudaErrorInvalidValue;
 }
 

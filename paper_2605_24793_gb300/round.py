@@ -40,7 +40,6 @@ class VerifyRound:
         self.w1, self.b1, self.w2 = w1.to(dev), b1.to(dev), w2.to(dev)
         self.b2 = float(b2)
         self.dims = C.attn_dims(self.q[0], self.k_pages[0], self.page_table)
-        self.ws_attn = C.new_attn_workspace(self.dims, self.max_ctx, dev)
         M = B * R
         self.ws_lm = C.new_lmhead_workspace(M, cfg.hidden, cfg.vocab, dev)
         nout = L if keep_attn else 1
@@ -70,8 +69,7 @@ class VerifyRound:
         pl = 0 if self.k_pages.shape[0] == 1 else l
         out = self.attn_out[l if self.attn_out.shape[0] > 1 else 0]
         return C.verify_attn(self.q[l], self.k_blk[l], self.v_blk[l], self.k_pages[pl],
-                             self.v_pages[pl], self.page_table, self.ctx_len, out, self.ws_attn,
-                             self.max_ctx)
+                             self.v_pages[pl], self.page_table, self.ctx_len, out, self.max_ctx)
 
     def lmhead(self):
         return C.lmhead_argmax_features(self.hidden, self.w, self.draft_for_row, self.argmax,

@@ -73,21 +73,17 @@ def test_verify_attention_matches_oracle(case):
     rng = np.random.default_rng(B * 1000 + R * 100 + Hq + D + sum(ctx))
     t = _paged_case(rng, B, R, Hq, Hkv, D, ctx, shuffled)
     max_ctx = max(ctx)
-    dims = C.attn_dims(t["q"], t["k_pages"], t["page_table"])
-    ws = C.new_attn_workspace(dims, max_ctx)
     out = torch.empty_like(t["q"])
     C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
-                  t["ctx_len"], out, ws, max_ctx)
+                  t["ctx_len"], out, max_ctx)
     ref = O.verify_attention(host(t["q"]), host(t["k_blk"]), host(t["v_blk"]), host(t["k_pages"]),
                              host(t["v_pages"]), t["table_np"], t["ctx_np"], 16)
     assert_close(host(out), ref, "attention")
-    # a second call on the same workspace (split counters must have been reset)
+    # a second call gives the same bits
     out2 = torch.empty_like(out)
     C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
-                  t["ctx_len"], out2, ws, max_ctx)
+                  t["ctx_len"], out2, max_ctx)
     assert torch.equal(out, out2)
-    nt = C.load_library().cospec_verify_attn_ticket_bytes(ctypes.byref(dims))
-    assert int(ws[:nt].sum()) == 0
 
 
 def test_verify_attention_split_count_does_not_change_result_beyond_tolerance():
@@ -96,11 +92,9 @@ def test_verify_attention_split_count_does_not_change_result_beyond_tolerance():
     ref = O.verify_attention(host(t["q"]), host(t["k_blk"]), host(t["v_blk"]), host(t["k_pages"]),
                              host(t["v_pages"]), t["table_np"], t["ctx_np"], 16)
     for max_ctx in (5000, t["table_np"].shape[1] * 16):     # different split plans
-        dims = C.attn_dims(t["q"], t["k_pages"], t["page_table"])
-        ws = C.new_attn_workspace(dims, max_ctx)
         out = torch.empty_like(t["q"])
         C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
-                      t["ctx_len"], out, ws, max_ctx)
+                      t["ctx_len"], out, max_ctx)
         assert_close(host(out), ref, f"attention max_ctx={max_ctx}")
 
 
@@ -110,11 +104,9 @@ def test_verify_attention_constant_values():
     t = _paged_case(rng, 2, 6, 32, 8, 128, [777, 3], True)
     t["v_pages"].fill_(0.375)
     t["v_blk"].fill_(0.375)
-    dims = C.attn_dims(t["q"], t["k_pages"], t["page_table"])
-    ws = C.new_attn_workspace(dims, 777)
     out = torch.empty_like(t["q"])
     C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
-                  t["ctx_len"], out, ws, 777)
+                  t["ctx_len"], out, 777)
     assert torch.all(out.float() == 0.375)
 
 
@@ -332,19 +324,16 @@ def test_block_size_one_round_is_greedy():
 def test_device_checks_set_error_bits_without_faulting():
     rng = np.random.default_rng(5)
     t = _paged_case(rng, 2, 6, 32, 8, 128, [100, 200], False)
-    dims = C.attn_dims(t["q"], t["k_pages"], t["page_table"])
-    ws = C.new_attn_workspace(dims, 200)
     out = torch.empty_like(t["q"])
     bad = t["page_table"].clone()
     bad[1, 3] = 10 ** 6                                    # page id outside the pool
     C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], bad, t["ctx_len"],
-                  out, ws, 200)
+                  out, 200)
     assert C.get_device_error() & C.DEVERR_PAGE
     long_ctx = torch.tensor([100, t["table_np"].shape[1] * 16 + 1], dtype=torch.int32, device="cuda")
     C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
-                  long_ctx, out, ws, 200)
+                  long_ctx, out, 200)
     assert C.get_device_error() & C.DEVERR_CTX
-    assert int(ws[:256].sum()) == 0                        # counters untouched by skipped units
     M, d, V = 4, 128, 256
     C.lmhead_argmax_features(bf16(rng.standard_normal((M, d))), bf16(rng.standard_normal((V, d))),
                              torch.tensor([0, V, -1, 5], dtype=torch.int32, device="cuda"),
