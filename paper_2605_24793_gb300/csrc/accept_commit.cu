@@ -23,6 +23,8 @@ __global__ void __launch_bounds__(128)
                        int32_t* __restrict__ emitted, int capacity, int* err) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b = blockIdx.x * 4 + warp;
+  griddep_wait();
+  griddep_launch_dependents();
   if (b >= B) return;
   const int R = K + 1;
   const bool act = lane < K;
@@ -53,6 +55,8 @@ __global__ void __launch_bounds__(128)
   __shared__ int s_len;
   const int l = blockIdx.x, b = blockIdx.y;
   const int R = a.K + 1;
+  griddep_wait();
+  griddep_launch_dependents();
   if (threadIdx.x < 32) {
     const int lane = threadIdx.x;
     const bool act = lane < a.K;
@@ -93,14 +97,11 @@ cudaError_t launch_accept_commit(const CommitArgs& a, int* err, cudaStream_t str
   if (a.B == 0) return cudaSuccess;
   const int capacity = a.max_pages * a.P;
   if (a.L > 0) {
-    commit_kernel<<<dim3(a.L, a.B), 128, 0, stream>>>(a, capacity, err);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_pdl(commit_kernel, dim3(a.L, a.B), dim3(128), 0, stream, a, capacity, err);
     if (e != cudaSuccess) return e;
   }
-  accept_scan_kernel<<<(a.B + 3) / 4, 128, 0, stream>>>(a.B, a.K, a.draft, a.argmax, a.accept,
-                                                        a.ctx_len, a.accept_len, a.emitted,
-                                                        capacity, err);
-  return cudaGetLastError();
+  return launch_pdl(accept_scan_kernel, dim3((a.B + 3) / 4), dim3(128), 0, stream, a.B, a.K,
+                    a.draft, a.argmax, a.accept, a.ctx_len, a.accept_len, a.emitted, capacity, err);
 }
 
 }  // namespace cospec

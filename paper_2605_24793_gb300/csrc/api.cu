@@ -64,9 +64,10 @@ bool encode_tensor_map_bf16(void* map, const void* base, int rank, const uint64_
       return false;
     fn = reinterpret_cast<EncodeTiledFn>(ptr);
   }
-  cuuint64_t d[3];
-  cuuint64_t st[2];
-  cuuint32_t bx[3], es[3];
+  if (rank < 1 || rank > 5) return false;
+  cuuint64_t d[5];
+  cuuint64_t st[4];
+  cuuint32_t bx[5], es[5];
   for (int i = 0; i < rank; ++i) {
     d[i] = dims[i];
     bx[i] = box[i];

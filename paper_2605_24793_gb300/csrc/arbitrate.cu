@@ -30,6 +30,8 @@ __global__ void __launch_bounds__(WARPS * 32)
   extern __shared__ float sm[];            // w1 [H][8], b1 [H], w2 [H] when mode == 0
   __shared__ float feat[WARPS][32][NF];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  griddep_wait();
+  griddep_launch_dependents();
   if (mode == 0) {
     for (int e = threadIdx.x; e < H * NF; e += blockDim.x) sm[e] = w1[e];
     for (int e = threadIdx.x; e < H; e += blockDim.x) {
@@ -114,9 +116,8 @@ cudaError_t launch_arbitrate(int B, int K, const int32_t* draft, const int32_t* 
     if (e != cudaSuccess) return e;
   }
   const int grid = (B + WARPS - 1) / WARPS;
-  arbitrate_kernel<<<grid, WARPS * 32, smem, stream>>>(B, K, draft, argmax, stats, H, w1, b1, w2,
-                                                         b2, lambda, mode, p_out, accept);
-  return cudaGetLastError();
+  return launch_pdl(arbitrate_kernel, dim3(grid), dim3(WARPS * 32), smem, stream, B, K, draft,
+                    argmax, stats, H, w1, b1, w2, b2, lambda, mode, p_out, accept);
 }
 
 }  // namespace cospec

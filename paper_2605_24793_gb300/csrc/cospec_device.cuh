@@ -59,6 +59,12 @@ CS_DEV void mma_16816(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
+// 2^x with the hardware approximation (relative error about 2^-22); -inf -> 0.
+CS_DEV float exp2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 CS_DEV uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
@@ -140,6 +146,15 @@ CS_DEV void tma_load_3d(uint32_t dst, const void* map, uint64_t* bar, int x, int
       : "memory");
 }
 
+CS_DEV void tma_load_4d(uint32_t dst, const void* map, uint64_t* bar, int x, int y, int z, int w,
+                        uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%3, %4, %5, %6}], [%2], %7;" ::"r"(dst),
+      "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y), "r"(z), "r"(w), "l"(policy)
+      : "memory");
+}
+
 // ---------------------------------------------------------------- clusters / DSMEM
 CS_DEV uint32_t cluster_ctarank() {
   uint32_t r;
@@ -161,6 +176,22 @@ CS_DEV uint32_t dsmem_map(uint32_t local, uint32_t rank) {
   uint32_t r;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
   return r;
+}
+// Bulk copy of `bytes` (multiple of 16) from this CTA's shared memory to
+// another CTA's shared memory in the cluster; completion is counted on the
+// destination CTA's mbarrier (cluster address).
+CS_DEV void bulk_copy_s2s(uint32_t dst_cluster, uint32_t src_cta, uint32_t bytes,
+                          uint32_t bar_cluster) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          dst_cluster),
+      "r"(src_cta), "r"(bytes), "r"(bar_cluster)
+      : "memory");
+}
+CS_DEV void dsmem_st_f4(uint32_t addr, float4 v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(v.x), "f"(v.y),
+               "f"(v.z), "f"(v.w)
+               : "memory");
 }
 CS_DEV float2 dsmem_ld_f2(uint32_t addr) {
   float2 v;
@@ -242,6 +273,14 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
          | (1u << 10)                    // B format: bf16
          | ((uint32_t)(N >> 3) << 17)    // N / 8
          | ((uint32_t)(M >> 4) << 24);   // M / 16
+}
+
+// Programmatic dependent launch: wait until the grids this one depends on
+// have completed and their writes are visible; allow the next grid in the
+// stream to begin launching (its own wait still orders its reads).
+CS_DEV void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+CS_DEV void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 CS_DEV void named_bar_sync(int id, int nthreads) {

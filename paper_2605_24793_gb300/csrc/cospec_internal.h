@@ -9,10 +9,29 @@
 
 namespace cospec {
 
+// Launch with programmatic stream serialization: the kernel may start while
+// the previous kernel of the stream finishes; it must call griddep_wait()
+// before reading anything an earlier kernel wrote.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t stream, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 int device_num_sms();
 int* device_error_word();  // device address of the error word of the current device
 
-// cuTensorMapEncodeTiled for a bf16 tensor (rank 2 or 3, innermost first),
+// cuTensorMapEncodeTiled for a bf16 tensor (rank 1..5, innermost first),
 // 128-byte swizzle, zero fill out of bounds.  dims/box in elements, strides
 // in bytes for dimensions 1..rank-1.
 bool encode_tensor_map_bf16(void* map, const void* base, int rank, const uint64_t* dims,

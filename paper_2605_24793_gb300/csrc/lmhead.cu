@@ -198,17 +198,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     tmem_alloc(tmem_holder, p.tmem_cols);
     tmem_relinquish();
   }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+  griddep_wait();                        // hidden rows may come from the previous kernel
   if (warp >= 2) {
     for (int c = tid - 64; c < p.n_mma; c += EPI_THREADS) {
       s_run[c] = make_float4(-INFINITY, -INFINITY, 0.f, 0.f);
       s_runi[c] = 0x7fffffff;
       s_draft[c] = (c < p.n_rows) ? p.draft_for_row[p.row0 + c] : -2;
     }
+    named_bar_sync(1, EPI_THREADS);
   }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem_base = *tmem_holder;
   const uint32_t idesc = idesc_bf16_f32(BM, p.n_mma);
 
   if (warp == 0) {
@@ -350,6 +352,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
       named_bar_sync(1, EPI_THREADS);
     }
+    griddep_launch_dependents();
     for (int col = etid; col < p.n_rows; col += EPI_THREADS) {
       p.part[(size_t)blockIdx.x * p.n_rows + col] = s_run[col];
       p.part_idx[(size_t)blockIdx.x * p.n_rows + col] = s_runi[col];
@@ -372,6 +375,8 @@ __global__ void __launch_bounds__(128) lmhead_reduce_kernel(const float4* part, 
                                                             int32_t* argmax, float* stats, int* err) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row = blockIdx.x * 4 + warp;
+  griddep_wait();
+  griddep_launch_dependents();
   if (row >= n_rows) return;
   Stat a = stat_identity();
   for (int c = lane; c < nparts; c += 32) {
@@ -465,12 +470,12 @@ cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
     p.stages = pl.stages;
     p.tmem_cols = tmem_cols;
     p.err = err;
-    lmhead_kernel<<<pl.grid, NUM_THREADS, pl.smem_bytes, stream>>>(map_w, map_h, p);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_pdl(lmhead_kernel, dim3(pl.grid), dim3(NUM_THREADS), pl.smem_bytes,
+                               stream, map_w, map_h, p);
     if (e != cudaSuccess) return e;
-    lmhead_reduce_kernel<<<(p.n_rows + 3) / 4, 128, 0, stream>>>(
-        part, part_idx, pl.grid, p.row0, p.n_rows, V, draft_for_row, argmax, stats, err);
-    e = cudaGetLastError();
+    e = launch_pdl(lmhead_reduce_kernel, dim3((p.n_rows + 3) / 4), dim3(128), 0, stream,
+                   (const float4*)part, (const int*)part_idx, pl.grid, p.row0, p.n_rows, V,
+                   draft_for_row, argmax, stats, err);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

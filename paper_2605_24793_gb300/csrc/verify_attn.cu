@@ -3,9 +3,10 @@
 //
 // One CTA owns (sequence b, KV head, KV split).  The KV range of a (b, head)
 // is split over the CTAs of one thread-block cluster; every CTA streams its
-// 64-token K/V tiles (4 pages) once with TMA tensor loads -- one thread
-// issues a 16-row x 128-byte box per page and half-row, 128B-swizzled, into
-// a 3-stage mbarrier ring -- and multiplies each tile against ALL query rows
+// 64-token K/V tiles (4 pages) once with TMA tensor loads -- one 3-D box per
+// page and tensor brings both 128-byte halves of the page's 16 rows,
+// 128B-swizzled, into a 3-stage mbarrier ring, the boxes of a tile issued
+// from several lanes of a producer warp at once -- and multiplies each tile against ALL query rows
 // that read this KV head (the G = Hq/Hkv heads of the group times the R block
 // rows, row index j*G + g).  Q.K^T and P.V run on bf16 tensor cores
 // (mma.m16n8k16, fp32 accumulation), the softmax is online in base 2.  The
@@ -26,7 +27,6 @@ namespace {
 constexpr int KT = 64;            // keys per cache tile (4 pages)
 constexpr int PAGE = 16;          // page size (fixed)
 constexpr int ROWB = 128;         // bytes of one swizzled smem row (64 bf16)
-constexpr int BOX_BYTES = PAGE * ROWB;  // one page x 64 columns
 constexpr int NSTAGE = 3;
 
 struct AttnParams {
@@ -43,24 +43,45 @@ struct AttnParams {
 template <int D, int MT, int WK>
 struct Layout {
   static constexpr int H = D / 64;                 // 128-byte halves of a key row
-  static constexpr int HALF = KT * ROWB;           // 8 KB: one half of a 64-key tile
-  static constexpr int STAGE = 2 * H * HALF;       // K halves then V halves
+  static constexpr int PAGEB = H * PAGE * ROWB;    // one page of K (or V): [H][16 rows][128 B]
+  static constexpr int KV = 4 * PAGEB;             // K (or V) of a 64-key tile
+  static constexpr int STAGE = 2 * KV;             // K then V
   static constexpr int NRP = MT * 16;
-  static constexpr int RED = (WK > 1) ? MT * WK * 16 * (D * 4 + 8) : 0;
-  static constexpr int PART_O = RED;               // [NRP][D] fp32
-  static constexpr int PART_ML = PART_O + NRP * D * 4;   // [NRP] (m, l)
-  static constexpr int PART_END = PART_ML + NRP * 8;
-  static constexpr int BAR = NSTAGE * STAGE;       // full[NSTAGE], empty[NSTAGE]
-  static constexpr int TOTAL = BAR + 2 * NSTAGE * 8;
+  static constexpr int PD = D + 8;                 // padded fp32 row of a partial (no bank conflicts)
+  static constexpr int ROWP = PD * 4;              // bytes of a partial row: O[D], (m, l), pad
+  static constexpr int RED = (WK > 1) ? MT * WK * 16 * ROWP : 0;
+  // Partials pushed by the cluster's CTAs land in RECV [S][rows per owner]
+  // (at most NRP rows in all); it overlaps RED and the ring, which are idle
+  // by then.  PART, this CTA's own partial [NRP rows], lies beyond both.
+  static constexpr int RECV = 0;
+  static constexpr bool CAN_SPLIT =
+      (RED > NRP * ROWP ? RED : NRP * ROWP) + NRP * ROWP <= NSTAGE * STAGE;   // else one CTA
+  static constexpr int PART = CAN_SPLIT ? (RED > NRP * ROWP ? RED : NRP * ROWP) : RED;
+  static constexpr int PART_END = PART + NRP * ROWP;
+  static constexpr int BAR = NSTAGE * STAGE;       // full[NSTAGE], empty[NSTAGE], block
+  static constexpr int BLK = BAR + (2 * NSTAGE + 2) * 8 + 1024;   // 1024-aligned block K/V
+  // the block region holds 2*H halves of KBR rows (KBR = 16 or 32, runtime)
+  static constexpr int blk_half(int kbr) { return kbr * ROWB; }
+  static constexpr int total(int kbr) { return BLK / 1024 * 1024 + 2 * H * kbr * ROWB; }
   static_assert(PART_END <= NSTAGE * STAGE, "partials must fit in the stage ring");
 };
 
+// Shared-memory byte offset of 16-byte chunk `ch` (of D/8) of key row `key`
+// in a region laid out as groups of 16 keys (`group_bytes` apart), each group
+// holding its 128-byte half rows half by half (`half_bytes` apart), every
+// 128-byte row swizzled by the TMA 128B pattern.
+CS_DEV uint32_t kv_off(int key, int ch, uint32_t group_bytes, uint32_t half_bytes) {
+  return (uint32_t)(key >> 4) * group_bytes + (uint32_t)(ch >> 3) * half_bytes +
+         (uint32_t)(key & 15) * ROWB + (uint32_t)(((ch & 7) ^ (key & 7)) * 16);
+}
+
 // Online-softmax update of one warp's 16 rows with NK keys held in shared
-// memory (K and V, 128B-swizzled rows of 64 bf16, halves `half_bytes`
-// apart).  Key k of the region sits at smem row key0 + k and has index
-// kidx0 + k for masking; row r sees key index <= lim_r.
+// memory (K and V regions laid out as in kv_off).  Key k of the region sits
+// at row key0 + k and has index kidx0 + k for masking; row r sees key index
+// <= lim_r.
 template <int D, int NK>
-CS_DEV void attend(uint32_t sk, uint32_t sv, uint32_t half_bytes, int key0, int kidx0,
+CS_DEV void attend(uint32_t sk, uint32_t sv, uint32_t group_bytes, uint32_t half_bytes,
+                   int key0, int kidx0,
                    bool need_mask, int lim0, int lim1, float scale_log2,
                    const uint32_t (&qf)[D / 16][4], float (&o)[D / 8][4], float& m0, float& m1,
                    float& l0, float& l1, int lane) {
@@ -74,8 +95,7 @@ CS_DEV void attend(uint32_t sk, uint32_t sv, uint32_t half_bytes, int key0, int 
 #pragma unroll
     for (int nt = 0; nt < NK / 8; ++nt) {
       const int key = key0 + nt * 8 + (lane & 7);
-      const uint32_t addr = sk + (uint32_t)(ch >> 3) * half_bytes + (uint32_t)key * ROWB +
-                            (uint32_t)(((ch & 7) ^ (key & 7)) * 16);
+      const uint32_t addr = sk + kv_off(key, ch, group_bytes, half_bytes);
       uint32_t b0, b1, b2, b3;
       ldsm_x4(addr, b0, b1, b2, b3);
       mma_16816(s[nt], qf[kk], b0, b1);
@@ -107,23 +127,26 @@ CS_DEV void attend(uint32_t sk, uint32_t sv, uint32_t half_bytes, int key0, int 
   const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
   const float base0 = (mn0 == -INFINITY) ? 0.f : mn0;
   const float base1 = (mn1 == -INFINITY) ? 0.f : mn1;
-  const float a0 = exp2f(m0 - base0), a1 = exp2f(m1 - base1);
+  const float a0 = exp2_approx(m0 - base0), a1 = exp2_approx(m1 - base1);
+  // Rescale the running output only when some row's maximum moved.
+  if (__any_sync(0xffffffffu, mn0 != m0 || mn1 != m1)) {
+    l0 *= a0;
+    l1 *= a1;
+#pragma unroll
+    for (int i = 0; i < D / 8; ++i) {
+      o[i][0] *= a0;
+      o[i][1] *= a0;
+      o[i][2] *= a1;
+      o[i][3] *= a1;
+    }
+  }
   m0 = mn0;
   m1 = mn1;
-  l0 *= a0;
-  l1 *= a1;
-#pragma unroll
-  for (int i = 0; i < D / 8; ++i) {
-    o[i][0] *= a0;
-    o[i][1] *= a0;
-    o[i][2] *= a1;
-    o[i][3] *= a1;
-  }
   uint32_t pf[NK / 16][4];
 #pragma unroll
   for (int nt = 0; nt < NK / 8; ++nt) {
-    const float p0 = exp2f(s[nt][0] - base0), p1 = exp2f(s[nt][1] - base0);
-    const float p2 = exp2f(s[nt][2] - base1), p3 = exp2f(s[nt][3] - base1);
+    const float p0 = exp2_approx(s[nt][0] - base0), p1 = exp2_approx(s[nt][1] - base0);
+    const float p2 = exp2_approx(s[nt][2] - base1), p3 = exp2_approx(s[nt][3] - base1);
     l0 += p0 + p1;
     l1 += p2 + p3;
     pf[nt / 2][(nt % 2) * 2 + 0] = pack_bf16(p0, p1);
@@ -135,8 +158,7 @@ CS_DEV void attend(uint32_t sk, uint32_t sv, uint32_t half_bytes, int key0, int 
 #pragma unroll
     for (int nd = 0; nd < D / 8; nd += 2) {
       const int ch = nd + (lane >> 4);
-      const uint32_t addr = sv + (uint32_t)(ch >> 3) * half_bytes + (uint32_t)key * ROWB +
-                            (uint32_t)(((ch & 7) ^ (key & 7)) * 16);
+      const uint32_t addr = sv + kv_off(key, ch, group_bytes, half_bytes);
       uint32_t b0, b1, b2, b3;
       ldsm_x4_t(addr, b0, b1, b2, b3);
       mma_16816(o[nd], pf[kk2], b0, b1);
@@ -158,7 +180,7 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
   constexpr int KW = KT / WK;            // cache keys of a tile handled by one warp
   constexpr int H = LY::H;
   constexpr int NRP = LY::NRP;
-  constexpr int SMAX = 16;
+  constexpr int PD = LY::PD;
   static_assert(KW % 16 == 0, "keys per warp must be a multiple of 16");
 
   extern __shared__ uint8_t smem_raw[];
@@ -166,11 +188,26 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + LY::BAR);
   uint64_t* empty = full + NSTAGE;
+  uint64_t* blk_full = empty + NSTAGE;
+  uint64_t* recv_bar = blk_full + 1;     // partials received from the cluster
+  uint8_t* blk_k = smem + LY::BLK / 1024 * 1024;          // block keys: 2*H halves of KBR rows
 
   const int S = (int)cluster_nctarank();
   const int rank = (int)cluster_ctarank();
   const int kvh = blockIdx.y, b = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+  if (tid == 0) {
+    for (int s2 = 0; s2 < NSTAGE; ++s2) {
+      mbar_init(&full[s2], 1);
+      mbar_init(&empty[s2], NWARPS);
+    }
+    mbar_init(blk_full, 1);
+    mbar_init(recv_bar, 1);
+    fence_barrier_init();
+  }
+  __syncthreads();
+  griddep_wait();                        // inputs may come from the previous kernel
 
   const int C = p.ctx_len[b];
   const bool bad = (C < 0) || (C > p.max_pages * PAGE);
@@ -180,19 +217,12 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
   const int tps = (nct + S - 1) / S;
   const int t_begin = min(nct, rank * tps);
   const int n = min(nct, t_begin + tps) - t_begin;
+  // The block's own keys go to the last CTA, which never has more cache tiles.
   const bool do_blk = !bad && rank == S - 1;
-  const int nv = n + (do_blk ? 1 : 0);                       // virtual tiles (block last)
+  const int nv = n;
   const int npages = (C + PAGE - 1) / PAGE;
   const int KBR = (p.R + 15) & ~15;                          // block keys padded to 16
-
-  if (tid == 0) {
-    for (int s2 = 0; s2 < NSTAGE; ++s2) {
-      mbar_init(&full[s2], 1);
-      mbar_init(&empty[s2], NWARPS);
-    }
-    fence_barrier_init();
-  }
-  __syncthreads();
+  uint8_t* blk_v = blk_k + H * KBR * ROWB;                   // each [H][KBR rows][128 B]
 
   float o[D / 8][4];
   float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
@@ -207,6 +237,13 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
       tma_prefetch_desc(&map_vp);
     }
     const uint64_t pol = l2_policy_evict_first();
+    if (do_blk && lane == 0) {
+      // one box per tensor: KBR rows from block row 0 of this head, both halves
+      // (rows past R belong to the next sequence or are zero-filled; masked)
+      mbar_arrive_expect_tx(blk_full, (uint32_t)(H * 2 * ROWB * KBR));   // KBR-row boxes
+      tma_load_4d(smem_u32(blk_k), &map_kb, blk_full, 0, b * p.R, 0, kvh, pol);
+      tma_load_4d(smem_u32(blk_v), &map_vb, blk_full, 0, b * p.R, 0, kvh, pol);
+    }
     const int* ptab = p.page_table + (size_t)b * p.max_pages + (size_t)t_begin * 4;
     const int my_pages = min(n * 4, npages - t_begin * 4);   // page-table entries of this CTA
     int pid = 0;
@@ -219,34 +256,21 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
       if (vt >= NSTAGE && !mbar_wait(&empty[st], (uint32_t)((vt / NSTAGE) - 1) & 1u))
         set_err(p.err, ERR_TIMEOUT);
       uint8_t* kb = smem + st * LY::STAGE;
-      uint8_t* vb = kb + H * LY::HALF;
-      if (vt < n) {
+      {
         const int np = min(4, npages - (t_begin + vt) * 4);
-        int page[4];
-#pragma unroll
-        for (int pg = 0; pg < 4; ++pg) page[pg] = __shfl_sync(0xffffffffu, pid, (vt & 7) * 4 + pg);
-        if (lane == 0) {
-          mbar_arrive_expect_tx(&full[st], (uint32_t)(np * H * 2 * BOX_BYTES));
-          for (int pg = 0; pg < np; ++pg) {
-            int pgid = page[pg];
-            if ((unsigned)pgid >= (unsigned)p.num_pages) {
-              set_err(p.err, ERR_PAGE);
-              pgid = 0;
-            }
-            const int y = (pgid * p.Hkv + kvh) * PAGE;
-#pragma unroll
-            for (int h = 0; h < H; ++h) {
-              tma_load_2d(smem_u32(kb + h * LY::HALF + pg * BOX_BYTES), &map_kp, &full[st], h * 64, y, pol);
-              tma_load_2d(smem_u32(vb + h * LY::HALF + pg * BOX_BYTES), &map_vp, &full[st], h * 64, y, pol);
-            }
+        // lanes 0..7: page lane/2 of the tile, K (even lane) or V (odd lane)
+        int pgid = __shfl_sync(0xffffffffu, pid, (vt & 7) * 4 + ((lane >> 1) & 3));
+        if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)(np * 2 * LY::PAGEB));
+        __syncwarp();
+        if (lane < 2 * np) {
+          if ((unsigned)pgid >= (unsigned)p.num_pages) {
+            set_err(p.err, ERR_PAGE);
+            pgid = 0;
           }
-        }
-      } else if (lane == 0) {
-        mbar_arrive_expect_tx(&full[st], (uint32_t)(H * 2 * ROWB * p.R));
-#pragma unroll
-        for (int h = 0; h < H; ++h) {
-          tma_load_3d(smem_u32(kb + h * LY::HALF), &map_kb, &full[st], h * 64, kvh, b * p.R, pol);
-          tma_load_3d(smem_u32(vb + h * LY::HALF), &map_vb, &full[st], h * 64, kvh, b * p.R, pol);
+          const int y = (pgid * p.Hkv + kvh) * PAGE;
+          const int pg = lane >> 1;
+          tma_load_3d(smem_u32(kb + (lane & 1) * LY::KV + pg * LY::PAGEB), (lane & 1) ? (const void*)&map_vp : (const void*)&map_kp,
+                      &full[st], 0, y, 0, pol);
         }
       }
       __syncwarp();
@@ -276,41 +300,51 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
 #pragma unroll
     for (int i = 0; i < D / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
 
-    for (int it = 0; it < nv; ++it) {
+    for (int it = 0; it < n; ++it) {
       const int st = it % NSTAGE;
       if (!mbar_wait(&full[st], (uint32_t)(it / NSTAGE) & 1u)) set_err(p.err, ERR_TIMEOUT);
       uint8_t* kb = smem + st * LY::STAGE;
-      uint8_t* vb = kb + H * LY::HALF;
-      const bool is_blk = (it == n);
+      uint8_t* vb = kb + LY::KV;
       // Rows past the valid keys of this tile may hold stale or unwritten
       // bytes: zero their V rows so that 0-weight keys contribute exactly 0.
-      const int valid_rows = is_blk ? p.R : min(KT, C - (t_begin + it) * KT);
-      const int zero_to = is_blk ? KBR : KT;
-      if (valid_rows < zero_to) {
-        const int nz = (zero_to - valid_rows) * H * (ROWB / 16);
+      const int valid_rows = min(KT, C - (t_begin + it) * KT);
+      if (valid_rows < KT) {
+        const int nz = (KT - valid_rows) * H * (ROWB / 16);
         for (int e = tid; e < nz; e += NTC) {
           const int row = valid_rows + e / (H * (ROWB / 16));
           const int rem = e % (H * (ROWB / 16));
-          *reinterpret_cast<uint4*>(vb + (rem / (ROWB / 16)) * LY::HALF + row * ROWB +
-                                    (rem % (ROWB / 16)) * 16) = make_uint4(0u, 0u, 0u, 0u);
+          *reinterpret_cast<uint4*>(vb + (row >> 4) * LY::PAGEB + (rem / (ROWB / 16)) * (PAGE * ROWB) +
+                                    (row & 15) * ROWB + (rem % (ROWB / 16)) * 16) =
+              make_uint4(0u, 0u, 0u, 0u);
         }
         fence_proxy_async_smem();
         named_bar_sync(1, NTC);
       }
-      if (!is_blk) {
-        const int kidx0 = (t_begin + it) * KT + wk * KW;
-        attend<D, KW>(smem_u32(kb), smem_u32(vb), LY::HALF, wk * KW, kidx0, valid_rows < KT,
-                      C - 1, C - 1, p.scale_log2, qf, o, m0, m1, l0, l1, lane);
-      } else if (wk == 0) {
-        if (KBR == 16)
-          attend<D, 16>(smem_u32(kb), smem_u32(vb), LY::HALF, 0, 0, true, j0, j1, p.scale_log2,
-                        qf, o, m0, m1, l0, l1, lane);
-        else
-          attend<D, 32>(smem_u32(kb), smem_u32(vb), LY::HALF, 0, 0, true, j0, j1, p.scale_log2,
-                        qf, o, m0, m1, l0, l1, lane);
-      }
+      const int kidx0 = (t_begin + it) * KT + wk * KW;
+      attend<D, KW>(smem_u32(kb), smem_u32(vb), LY::PAGEB, PAGE * ROWB, wk * KW, kidx0,
+                    valid_rows < KT, C - 1, C - 1, p.scale_log2, qf, o, m0, m1, l0, l1, lane);
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty[st]);
+    }
+    if (do_blk) {
+      if (!mbar_wait(blk_full, 0)) set_err(p.err, ERR_TIMEOUT);
+      // rows R..KBR-1 of the block region were never written: zero their V
+      const int nz = (KBR - p.R) * H * (ROWB / 16);
+      for (int e = tid; e < nz; e += NTC) {
+        const int row = p.R + e / (H * (ROWB / 16));
+        const int rem = e % (H * (ROWB / 16));
+        *reinterpret_cast<uint4*>(blk_v + (rem / (ROWB / 16)) * KBR * ROWB + row * ROWB +
+                                  (rem % (ROWB / 16)) * 16) = make_uint4(0u, 0u, 0u, 0u);
+      }
+      named_bar_sync(1, NTC);
+      if (wk == 0) {
+        if (KBR == 16)
+          attend<D, 16>(smem_u32(blk_k), smem_u32(blk_v), PAGE * ROWB, 16 * ROWB, 0, 0, true, j0,
+                        j1, p.scale_log2, qf, o, m0, m1, l0, l1, lane);
+        else
+          attend<D, 32>(smem_u32(blk_k), smem_u32(blk_v), PAGE * ROWB, 32 * ROWB, 0, 0, true, j0,
+                        j1, p.scale_log2, qf, o, m0, m1, l0, l1, lane);
+      }
     }
     // After a timed-out wait a copy may still be in flight: wait (bounded)
     // for the last fill of every stage before the ring is reused.
@@ -319,44 +353,45 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
         const int last = st + ((nv - 1 - st) / NSTAGE) * NSTAGE;
         mbar_wait(&full[st], (uint32_t)(last / NSTAGE) & 1u);
       }
+      if (do_blk) mbar_wait(blk_full, 0);
     }
     l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
     l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
     l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
     l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
   }
+  griddep_launch_dependents();
   __syncthreads();
 
   // CTA partial: rows of every warp, key groups merged (stage ring reused).
-  float* part_o = reinterpret_cast<float*>(smem + LY::PART_O);
-  float2* part_ml = reinterpret_cast<float2*>(smem + LY::PART_ML);
+  // A partial row holds O[0..D) then (m, l) at D, D+1 (fp32, padded to PD).
+  float* part = reinterpret_cast<float*>(smem + LY::PART);
   if constexpr (WK == 1) {
     if (warp < NWARPS) {
 #pragma unroll
       for (int nd = 0; nd < D / 8; ++nd) {
         const int col = nd * 8 + 2 * c4;
-        *reinterpret_cast<float2*>(part_o + r0 * D + col) = make_float2(o[nd][0], o[nd][1]);
-        *reinterpret_cast<float2*>(part_o + r1 * D + col) = make_float2(o[nd][2], o[nd][3]);
+        *reinterpret_cast<float2*>(part + r0 * PD + col) = make_float2(o[nd][0], o[nd][1]);
+        *reinterpret_cast<float2*>(part + r1 * PD + col) = make_float2(o[nd][2], o[nd][3]);
       }
       if (c4 == 0) {
-        part_ml[r0] = make_float2(m0, l0);
-        part_ml[r1] = make_float2(m1, l1);
+        *reinterpret_cast<float2*>(part + r0 * PD + D) = make_float2(m0, l0);
+        *reinterpret_cast<float2*>(part + r1 * PD + D) = make_float2(m1, l1);
       }
     }
   } else {
-    float* red_o = reinterpret_cast<float*>(smem);                        // [NWARPS][16][D]
-    float2* red_ml = reinterpret_cast<float2*>(red_o + NWARPS * 16 * D);  // [NWARPS][16]
+    float* red = reinterpret_cast<float*>(smem);                          // [NWARPS][16][PD]
     if (warp < NWARPS) {
-      float* wo = red_o + warp * 16 * D;
+      float* wo = red + warp * 16 * PD;
 #pragma unroll
       for (int nd = 0; nd < D / 8; ++nd) {
         const int col = nd * 8 + 2 * c4;
-        *reinterpret_cast<float2*>(wo + g_row * D + col) = make_float2(o[nd][0], o[nd][1]);
-        *reinterpret_cast<float2*>(wo + (g_row + 8) * D + col) = make_float2(o[nd][2], o[nd][3]);
+        *reinterpret_cast<float2*>(wo + g_row * PD + col) = make_float2(o[nd][0], o[nd][1]);
+        *reinterpret_cast<float2*>(wo + (g_row + 8) * PD + col) = make_float2(o[nd][2], o[nd][3]);
       }
       if (c4 == 0) {
-        red_ml[warp * 16 + g_row] = make_float2(m0, l0);
-        red_ml[warp * 16 + g_row + 8] = make_float2(m1, l1);
+        *reinterpret_cast<float2*>(wo + g_row * PD + D) = make_float2(m0, l0);
+        *reinterpret_cast<float2*>(wo + (g_row + 8) * PD + D) = make_float2(m1, l1);
       }
     }
     __syncthreads();
@@ -365,59 +400,68 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
       const int rt = r / 16, ri = r % 16;
       float M = -INFINITY;
 #pragma unroll
-      for (int w = 0; w < WK; ++w) M = fmaxf(M, red_ml[(rt * WK + w) * 16 + ri].x);
+      for (int w = 0; w < WK; ++w) M = fmaxf(M, red[((rt * WK + w) * 16 + ri) * PD + D]);
       float L = 0.f;
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
       if (M != -INFINITY) {
 #pragma unroll
         for (int w = 0; w < WK; ++w) {
-          const float2 ml = red_ml[(rt * WK + w) * 16 + ri];
-          const float sc = exp2f(ml.x - M);
-          L += ml.y * sc;
-          const float4 v = *reinterpret_cast<const float4*>(red_o + ((rt * WK + w) * 16 + ri) * D + c);
+          const float* wr_ = red + ((rt * WK + w) * 16 + ri) * PD;
+          const float sc = exp2_approx(wr_[D] - M);
+          L += wr_[D + 1] * sc;
+          const float4 v = *reinterpret_cast<const float4*>(wr_ + c);
           acc.x += v.x * sc;
           acc.y += v.y * sc;
           acc.z += v.z * sc;
           acc.w += v.w * sc;
         }
       }
-      *reinterpret_cast<float4*>(part_o + r * D + c) = acc;
-      if (c == 0) part_ml[r] = make_float2(M, L);
+      *reinterpret_cast<float4*>(part + r * PD + c) = acc;
+      if (c == 0) *reinterpret_cast<float2*>(part + r * PD + D) = make_float2(M, L);
     }
   }
+  fence_proxy_async_smem();              // the bulk copies below read `part`
+  __syncthreads();
 
-  // Merge the S partials of the cluster; CTA `rank` finishes every S-th chunk.
-  // All remote loads of an element are issued before any is consumed.
-  cluster_sync();
-  const uint32_t po = smem_u32(part_o), pml = smem_u32(part_ml);
-  for (int e = rank * NTT + tid; e < p.NR * (D / 4); e += S * NTT) {
-    const int r = e / (D / 4), c = (e % (D / 4)) * 4;
-    float2 ml[SMAX];
-    float4 v[SMAX];
-#pragma unroll
-    for (int s2 = 0; s2 < SMAX; ++s2) {
-      if (s2 < S) {
-        ml[s2] = dsmem_ld_f2(dsmem_map(pml + r * 8, s2));
-        v[s2] = dsmem_ld_f4(dsmem_map(po + (uint32_t)(r * D + c) * 4, s2));
-      }
+  // Reduce-scatter over the cluster: owner o finishes rows [o*rpo, (o+1)*rpo).
+  // Each CTA sends its partial rows to their owners with one bulk shared-
+  // to-shared copy per owner (thread-level remote accesses are slow); the
+  // owner merges the S received copies from its own shared memory.
+  const int rpo = (p.NR + S - 1) / S;
+  const float* src = part;
+  if (S > 1) {
+    if (tid == 0) mbar_arrive_expect_tx(recv_bar, (uint32_t)(S * rpo * LY::ROWP));
+    cluster_sync();                      // peers' rings / reduction buffers are idle now
+    float* recv = reinterpret_cast<float*>(smem + LY::RECV);   // [S][rpo][PD] at each owner
+    if (tid == 0) {
+      const uint32_t recv_u = smem_u32(recv), bar_u = smem_u32(recv_bar);
+      for (int o = 0; o < S; ++o)
+        bulk_copy_s2s(dsmem_map(recv_u + (uint32_t)(rank * rpo * LY::ROWP), (uint32_t)o),
+                      smem_u32(part + o * rpo * PD), (uint32_t)(rpo * LY::ROWP),
+                      dsmem_map(bar_u, (uint32_t)o));
     }
+    if (!mbar_wait(recv_bar, 0)) set_err(p.err, ERR_TIMEOUT);
+    src = recv;
+  }
+  const int row0 = rank * rpo;
+  for (int e = tid; e < rpo * (D / 4); e += NTT) {
+    const int rr = e / (D / 4), c = (e % (D / 4)) * 4;
+    const int r = row0 + rr;
+    if (r >= p.NR) break;
     float M = -INFINITY;
-#pragma unroll
-    for (int s2 = 0; s2 < SMAX; ++s2)
-      if (s2 < S) M = fmaxf(M, ml[s2].x);
+    for (int s2 = 0; s2 < S; ++s2) M = fmaxf(M, src[(s2 * rpo + rr) * PD + D]);
     float L = 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     if (M != -INFINITY) {
-#pragma unroll
-      for (int s2 = 0; s2 < SMAX; ++s2) {
-        if (s2 < S) {
-          const float sc = (ml[s2].x == -INFINITY) ? 0.f : exp2f(ml[s2].x - M);
-          L += ml[s2].y * sc;
-          acc.x += v[s2].x * sc;
-          acc.y += v[s2].y * sc;
-          acc.z += v[s2].z * sc;
-          acc.w += v[s2].w * sc;
-        }
+      for (int s2 = 0; s2 < S; ++s2) {
+        const float* pr = src + (s2 * rpo + rr) * PD;
+        const float sc = exp2_approx(pr[D] - M);
+        L += pr[D + 1] * sc;
+        const float4 v = *reinterpret_cast<const float4*>(pr + c);
+        acc.x += v.x * sc;
+        acc.y += v.y * sc;
+        acc.z += v.z * sc;
+        acc.w += v.w * sc;
       }
     }
     const float inv = (L > 0.f) ? 1.f / L : 0.f;
@@ -428,20 +472,22 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
     pk.y = pack_bf16(acc.z * inv, acc.w * inv);
     *reinterpret_cast<uint2*>(dst) = pk;
   }
-  cluster_sync();   // peers may still read this CTA's partial until here
+  if (S > 1) cluster_sync();             // every copy out of this CTA has landed
 }
+
 
 template <int D, int MT, int WK>
 cudaError_t launch_t(const CUtensorMap* maps, const AttnParams& p, int S, int B, int Hkv,
                      cudaStream_t stream) {
   using LY = Layout<D, MT, WK>;
-  const size_t smem = LY::TOTAL + 1024;
+  const size_t smem = LY::total(p.R <= 16 ? 16 : 32) + 1024;
   static bool configured[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
   auto kern = verify_attn_kernel<D, MT, WK>;
   if (dev < 64 && !configured[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)(LY::total(32) + 1024));
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
@@ -452,13 +498,15 @@ cudaError_t launch_t(const CUtensorMap* maps, const AttnParams& p, int S, int B,
   cfg.blockDim = dim3(MT * WK * 32 + 32, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = S;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], maps[2], maps[3], p);
 }
 
@@ -466,12 +514,12 @@ template <int D, int MT, int WK>
 int max_cluster_t(int S, int Hkv, int B) {
   using LY = Layout<D, MT, WK>;
   auto kern = verify_attn_kernel<D, MT, WK>;
-  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(LY::TOTAL + 1024));
+  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(LY::total(32) + 1024));
   cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(S, Hkv, B);
   cfg.blockDim = dim3(MT * WK * 32 + 32, 1, 1);
-  cfg.dynamicSmemBytes = LY::TOTAL + 1024;
+  cfg.dynamicSmemBytes = LY::total(16) + 1024;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = S;
@@ -512,6 +560,7 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
   const long long want = (4LL * num_sms + units - 1) / (units > 0 ? units : 1);
   int S = 1;
   while (S < 16 && S < want && (S * 2) * 4 <= tiles) S *= 2;
+  if (pl.mt == 8) S = 1;   // the 128-row partials leave no room to receive a cluster's pushes
   pl.cluster = S;
   pl.tiles_per_split = (tiles + S - 1) / S;
   pl.max_splits = S;
@@ -529,18 +578,22 @@ int attn_max_active_clusters(int D, int mt, int wk, int S, int Hkv, int B) {
 
 cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& pl, int* err,
                                cudaStream_t stream) {
+  // Pool as {64 columns, rows, half}: a {64, 16, H} box is one page of one
+  // head, both 128-byte halves, landing as [half][16 rows][128 B].
   CUtensorMap maps[4];
+  const int H = a.D / 64;
   const uint64_t pool_rows = (uint64_t)a.num_pages * a.Hkv * PAGE;
-  const uint64_t dp[2] = {(uint64_t)a.D, pool_rows};
-  const uint64_t sp[1] = {(uint64_t)a.D * 2};
-  const uint32_t bp[2] = {64, PAGE};
-  const uint64_t db[3] = {(uint64_t)a.D, (uint64_t)a.Hkv, (uint64_t)a.B * a.R};
-  const uint64_t sb[2] = {(uint64_t)a.D * 2, (uint64_t)a.Hkv * a.D * 2};
-  const uint32_t bb[3] = {64, 1, (uint32_t)a.R};
-  if (!encode_tensor_map_bf16(&maps[0], a.k_pages, 2, dp, sp, bp) ||
-      !encode_tensor_map_bf16(&maps[1], a.v_pages, 2, dp, sp, bp) ||
-      !encode_tensor_map_bf16(&maps[2], a.k_blk, 3, db, sb, bb) ||
-      !encode_tensor_map_bf16(&maps[3], a.v_blk, 3, db, sb, bb))
+  const uint64_t dp[3] = {64, pool_rows, (uint64_t)H};
+  const uint64_t sp[2] = {(uint64_t)a.D * 2, 128};
+  const uint32_t bp[3] = {64, PAGE, (uint32_t)H};
+  // Block K/V as {64 columns, batch*rows, half, head}: one box per (b, head).
+  const uint64_t db[4] = {64, (uint64_t)a.B * a.R, (uint64_t)H, (uint64_t)a.Hkv};
+  const uint64_t sb[3] = {(uint64_t)a.Hkv * a.D * 2, 128, (uint64_t)a.D * 2};
+  const uint32_t bb[4] = {64, (uint32_t)(a.R <= 16 ? 16 : 32), (uint32_t)H, 1};
+  if (!encode_tensor_map_bf16(&maps[0], a.k_pages, 3, dp, sp, bp) ||
+      !encode_tensor_map_bf16(&maps[1], a.v_pages, 3, dp, sp, bp) ||
+      !encode_tensor_map_bf16(&maps[2], a.k_blk, 4, db, sb, bb) ||
+      !encode_tensor_map_bf16(&maps[3], a.v_blk, 4, db, sb, bb))
     return cudaErrorInvalidValue;
   AttnParams p{};
   p.q = a.q;
