@@ -148,6 +148,28 @@ COSPEC_API int cospec_lmhead_argmax_features(int M, int d, int V, const uint16_t
                                              int32_t* argmax, float* stats, void* ws,
                                              size_t ws_bytes, void* stream);
 
+/* Same computation and outputs as cospec_lmhead_argmax_features, for callers
+ * that cannot allocate device memory or hand this library a workspace -- for
+ * example a serving engine that reserves nearly all HBM for its KV cache and
+ * allows no allocation while decoding, or a plug-in inside a framework that
+ * owns the device's memory.  (The paper has no counterpart; this is an
+ * interface convenience of this library.)
+ *
+ * The per-CTA partial statistics go to a fixed 1.25 MiB scratch array
+ * compiled into the library, present on every GPU that loads it until the
+ * process exits; nothing is allocated and nothing needs clearing, since each
+ * call overwrites the scratch it reads.  The first call on each device looks
+ * up the scratch's device address (cudaGetSymbolAddress); make that first
+ * call before any stream capture.  All calls share the one array, so calls
+ * whose execution overlaps on the GPU (other streams, other host threads)
+ * race and give wrong results: keep them ordered on one stream.
+ * Limits: M <= 512 rows per call and at most 256 persistent CTAs (SMs);
+ * larger requests return COSPEC_ERR_UNSUPPORTED. */
+COSPEC_API int cospec_lmhead_argmax_features_noalloc(int M, int d, int V, const uint16_t* hidden,
+                                                     const uint16_t* w,
+                                                     const int32_t* draft_for_row,
+                                                     int32_t* argmax, float* stats, void* stream);
+
 /* ------------------------------------------------------------------------ */
 /* 3. Arbitration at draft/target mismatches (Sec. 3.3).
  *

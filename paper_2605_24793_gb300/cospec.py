@@ -21,7 +21,7 @@ DEVERR_PAGE, DEVERR_CTX, DEVERR_TOKEN, DEVERR_TIMEOUT = 1, 2, 4, 8
 
 EXPORTED = ("cospec_status_string", "cospec_get_device_error", "cospec_num_sms",
             "cospec_verify_attn", "cospec_lmhead_workspace", "cospec_lmhead_argmax_features",
-            "cospec_arbitrate", "cospec_accept_commit")
+            "cospec_arbitrate", "cospec_accept_commit", "cospec_lmhead_argmax_features_noalloc")
 
 
 class AttnDims(ctypes.Structure):
@@ -56,6 +56,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "cospec_verify_attn": (_i, [_PDIMS, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
         "cospec_lmhead_workspace": (_sz, [_i, _i, _i]),
         "cospec_lmhead_argmax_features": (_i, [_i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+        "cospec_lmhead_argmax_features_noalloc": (_i, [_i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp]),
         "cospec_arbitrate": (_i, [_i, _i, _vp, _vp, _vp, _i, _vp, _vp, _vp, _f, _f, _i, _vp, _vp, _vp]),
         "cospec_accept_commit": (_i, [_i, _i, _i, _PDIMS, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                       ctypes.c_longlong, _vp, _vp, _vp, _vp, _vp]),
@@ -152,6 +153,25 @@ def lmhead_argmax_features(hidden, w, draft_for_row, argmax, stats, ws, stream=N
     _check(load_library().cospec_lmhead_argmax_features(
         M, d, V, _ptr(hidden), _ptr(w), _ptr(draft_for_row), _ptr(argmax), _ptr(stats), _ptr(ws),
         ws.numel(), _stream(stream)))
+    return argmax, stats
+
+
+def lmhead_argmax_features_noalloc(hidden, w, draft_for_row, argmax, stats, stream=None):
+    """The LM-head call without a workspace, for callers that cannot allocate
+    device memory: partials go to a fixed scratch array inside the library
+    (at most 512 rows per call; calls must not overlap on the GPU)."""
+    _req(hidden, torch.bfloat16, "hidden", 2)
+    _req(w, torch.bfloat16, "w", 2)
+    _req(draft_for_row, torch.int32, "draft_for_row", 1)
+    _req(argmax, torch.int32, "argmax", 1)
+    _req(stats, torch.float32, "stats", 2)
+    M, d = hidden.shape
+    V = w.shape[0]
+    if w.shape[1] != d or draft_for_row.numel() != M or argmax.numel() != M or tuple(stats.shape) != (M, 5):
+        raise ValueError("inconsistent LM-head shapes")
+    _check(load_library().cospec_lmhead_argmax_features_noalloc(
+        M, d, V, _ptr(hidden), _ptr(w), _ptr(draft_for_row), _ptr(argmax), _ptr(stats),
+        _stream(stream)))
     return argmax, stats
 
 

@@ -19,6 +19,7 @@
 #include <cuda.h>
 #include <math.h>
 
+#include "../../include/cospec.h"
 #include "cospec_device.cuh"
 #include "cospec_internal.h"
 
@@ -481,4 +482,105 @@ cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
   return cudaSuccess;
 }
 
+// ---------------------------------------------------------------------------
+// Allocation-free variant of the LM-head call.
+//
+// Some callers cannot give this library device memory: a serving engine that
+// reserves almost all of HBM for its KV cache up front and forbids any other
+// allocation during decoding, or a plug-in running inside a host framework
+// that owns the device's memory and exposes no workspace.  For them the
+// per-CTA partial statistics live in one fixed scratch array compiled into
+// the library (resident on every GPU that loads it, until the process exits)
+// instead of a caller-provided workspace.
+//
+// The array below is a device symbol: in host code its name is only a
+// stand-in, never a device address.  Its address is looked up with
+// cudaGetSymbolAddress once per device, on that device's first call.
+namespace {
+
+constexpr int NOALLOC_MAX_CTAS = 256;                 // persistent CTAs (one per SM)
+constexpr int NOALLOC_MAX_M = 512;                    // rows per call (two 256-row passes)
+constexpr size_t NOALLOC_ENTRIES = (size_t)NOALLOC_MAX_CTAS * MAX_ROWS;
+// [NOALLOC_ENTRIES] float4 (m, second, s, t) then [NOALLOC_ENTRIES] int (argmax)
+static __device__ __align__(256) unsigned char g_lmhead_scratch[NOALLOC_ENTRIES * (sizeof(float4) + sizeof(int))];
+
+void* g_scratch_addr[64] = {nullptr};
+
+void* scratch_address() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  if (!g_scratch_addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_lmhead_scratch) != cudaSuccess) return nullptr;
+    g_scratch_addr[dev] = p;
+  }
+  return g_scratch_addr[dev];
+}
+
+}  // namespace
+
 }  // namespace cospec
+
+extern "C" COSPEC_API int cospec_lmhead_argmax_features_noalloc(
+    int M, int d, int V, const uint16_t* hidden, const uint16_t* w, const int32_t* draft_for_row,
+    int32_t* argmax, float* stats, void* stream) {
+  using namespace cospec;
+  if (M < 0 || d <= 0 || V <= 0) return COSPEC_ERR_INVALID_ARG;
+  if (M == 0) return COSPEC_OK;
+  if (!hidden || !w || !draft_for_row || !argmax || !stats) return COSPEC_ERR_INVALID_ARG;
+  if (d % 64 != 0 || (long long)V > 0x7fffff00LL) return COSPEC_ERR_UNSUPPORTED;
+  if ((reinterpret_cast<uintptr_t>(hidden) & 15u) || (reinterpret_cast<uintptr_t>(w) & 15u))
+    return COSPEC_ERR_INVALID_ARG;
+  if (M > NOALLOC_MAX_M) return COSPEC_ERR_UNSUPPORTED;          // beyond the fixed scratch
+  const int sms = device_num_sms();
+  if (sms <= 0) return COSPEC_ERR_CUDA;
+  const LmheadPlan pl = plan_lmhead(M, d, V, sms);
+  if (pl.grid > NOALLOC_MAX_CTAS) return COSPEC_ERR_UNSUPPORTED;  // beyond the fixed scratch
+  void* scratch = scratch_address();
+  int* err = device_error_word();
+  if (!scratch || !err) return COSPEC_ERR_CUDA;
+  float4* part = static_cast<float4*>(scratch);
+  int* part_idx = reinterpret_cast<int*>(part + NOALLOC_ENTRIES);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  CUtensorMap map_w, map_h;
+  if (!make_map(&map_w, w, (uint64_t)V, (uint64_t)d, BM) ||
+      !make_map(&map_h, hidden, (uint64_t)M, (uint64_t)d, (uint32_t)pl.n_mma))
+    return COSPEC_ERR_CUDA;
+  static bool configured[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 64 && !configured[dev]) {
+    if (cudaFuncSetAttribute(lmhead_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             227 * 1024) != cudaSuccess)
+      return COSPEC_ERR_CUDA;
+    configured[dev] = true;
+  }
+  uint32_t tmem_cols = 32;
+  while (tmem_cols < (uint32_t)(2 * pl.n_mma)) tmem_cols <<= 1;
+  // Each pass overwrites every scratch entry its merge kernel reads, so the
+  // contents left by an earlier call never need clearing.
+  for (int pass = 0; pass < pl.passes; ++pass) {
+    LmParams p{};
+    p.draft_for_row = draft_for_row;
+    p.stats = stats;
+    p.part = part;
+    p.part_idx = part_idx;
+    p.row0 = pass * MAX_ROWS;
+    p.n_rows = (M - p.row0) < MAX_ROWS ? (M - p.row0) : MAX_ROWS;
+    p.n_mma = pl.n_mma;
+    p.d = d;
+    p.V = V;
+    p.num_tiles = pl.num_tiles;
+    p.stages = pl.stages;
+    p.tmem_cols = tmem_cols;
+    p.err = err;
+    if (launch_pdl(lmhead_kernel, dim3(pl.grid), dim3(NUM_THREADS), pl.smem_bytes, st, map_w,
+                   map_h, p) != cudaSuccess)
+      return COSPEC_ERR_CUDA;
+    if (launch_pdl(lmhead_reduce_kernel, dim3((p.n_rows + 3) / 4), dim3(128), 0, st,
+                   (const float4*)part, (const int*)part_idx, pl.grid, p.row0, p.n_rows, V,
+                   draft_for_row, argmax, stats, err) != cudaSuccess)
+      return COSPEC_ERR_CUDA;
+  }
+  return COSPEC_OK;
+}
