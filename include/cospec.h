@@ -113,7 +113,14 @@ typedef struct {
   int max_pages_per_seq;
   int num_pages;
   float softmax_scale;   /* <= 0 selects 1/sqrt(head_dim) */
+  int flags;             /* COSPEC_ATTN_* bits, 0 by default */
 } cospec_attn_dims;
+
+/* The call may start reading ctx_len, page_table and the cached pages before
+ * the kernel queued just before it on the stream has finished: set it only
+ * when that kernel writes none of them (e.g. between the layers of one
+ * round, where only q / k_blk / v_blk come from the previous layer). */
+#define COSPEC_ATTN_KV_STABLE 1
 
 COSPEC_API int cospec_verify_attn(const cospec_attn_dims* dims, int max_ctx,
                                   const uint16_t* q, const uint16_t* k_blk, const uint16_t* v_blk,

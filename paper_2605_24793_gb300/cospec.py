@@ -28,7 +28,11 @@ class AttnDims(ctypes.Structure):
     _fields_ = [("batch", ctypes.c_int), ("rows", ctypes.c_int), ("num_q_heads", ctypes.c_int),
                 ("num_kv_heads", ctypes.c_int), ("head_dim", ctypes.c_int),
                 ("page_size", ctypes.c_int), ("max_pages_per_seq", ctypes.c_int),
-                ("num_pages", ctypes.c_int), ("softmax_scale", ctypes.c_float)]
+                ("num_pages", ctypes.c_int), ("softmax_scale", ctypes.c_float),
+                ("flags", ctypes.c_int)]
+
+
+ATTN_KV_STABLE = 1
 
 
 class CospecError(RuntimeError):
@@ -97,13 +101,13 @@ def _req(t: torch.Tensor, dtype, name: str, ndim: Optional[int] = None):
 
 
 def attn_dims(q: torch.Tensor, k_pages: torch.Tensor, page_table: torch.Tensor,
-              softmax_scale: float = 0.0) -> AttnDims:
+              softmax_scale: float = 0.0, flags: int = 0) -> AttnDims:
     """Geometry of one verify-attention call from q [B,R,Hq,D], the layer's
     pool [num_pages,Hkv,P,D] and the page table [B,max_pages]."""
     B, R, Hq, D = q.shape
     num_pages, Hkv, P, D2 = k_pages.shape[-4:]
     assert D2 == D
-    return AttnDims(B, R, Hq, Hkv, D, P, page_table.shape[1], num_pages, softmax_scale)
+    return AttnDims(B, R, Hq, Hkv, D, P, page_table.shape[1], num_pages, softmax_scale, flags)
 
 
 def num_sms() -> int:
@@ -111,14 +115,16 @@ def num_sms() -> int:
 
 
 def verify_attn(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len, out, max_ctx,
-                softmax_scale: float = 0.0, stream=None) -> torch.Tensor:
-    """Verify attention of one layer (Sec. 3.1, Eq. 2).  See include/cospec.h."""
+                softmax_scale: float = 0.0, stream=None, kv_stable: bool = False) -> torch.Tensor:
+    """Verify attention of one layer (Sec. 3.1, Eq. 2).  See include/cospec.h.
+    ``kv_stable``: the kernel queued just before writes neither ctx_len, the
+    page table nor the cached pages (COSPEC_ATTN_KV_STABLE)."""
     for t, n in ((q, "q"), (k_blk, "k_blk"), (v_blk, "v_blk"), (k_pages, "k_pages"),
                  (v_pages, "v_pages"), (out, "out")):
         _req(t, torch.bfloat16, n)
     _req(page_table, torch.int32, "page_table", 2)
     _req(ctx_len, torch.int32, "ctx_len", 1)
-    dims = attn_dims(q, k_pages, page_table, softmax_scale)
+    dims = attn_dims(q, k_pages, page_table, softmax_scale, ATTN_KV_STABLE if kv_stable else 0)
     if tuple(k_blk.shape) != (dims.batch, dims.rows, dims.num_kv_heads, dims.head_dim):
         raise ValueError("k_blk shape does not match q / pages")
     if out.shape != q.shape:
@@ -223,7 +229,7 @@ def accept_commit(draft, argmax, accept, k_blk, v_blk, k_pages, v_pages, page_ta
     # a single pool shared by every layer is passed with layer stride 0
     layer_stride = 0 if (k_pages.shape[0] == 1 and L > 1) else int(k_pages.stride(0))
     dims = AttnDims(B, K + 1, 0, k_pages.shape[2], k_pages.shape[4], k_pages.shape[3],
-                    page_table.shape[1], k_pages.shape[1], 0.0)
+                    page_table.shape[1], k_pages.shape[1], 0.0, 0)
     dims.num_q_heads = dims.num_kv_heads
     _check(load_library().cospec_accept_commit(
         B, K, L, ctypes.byref(dims), _ptr(draft), _ptr(argmax), _ptr(accept), _ptr(k_blk),

@@ -130,6 +130,7 @@ static int check_attn_dims(const cospec_attn_dims* d) {
     return COSPEC_ERR_INVALID_ARG;
   if (d->num_q_heads % d->num_kv_heads != 0) return COSPEC_ERR_INVALID_ARG;
   if (isnan(d->softmax_scale) || isinf(d->softmax_scale)) return COSPEC_ERR_INVALID_ARG;
+  if (d->flags & ~COSPEC_ATTN_KV_STABLE) return COSPEC_ERR_INVALID_ARG;
   if (d->head_dim != 64 && d->head_dim != 128) return COSPEC_ERR_UNSUPPORTED;
   if (d->page_size != 16) return COSPEC_ERR_UNSUPPORTED;
   if (d->rows > 32) return COSPEC_ERR_UNSUPPORTED;
@@ -194,6 +195,7 @@ COSPEC_API int cospec_verify_attn(const cospec_attn_dims* d, int max_ctx, const 
   a.num_pages = d->num_pages;
   a.scale = d->softmax_scale > 0.f ? d->softmax_scale : 1.0f / sqrtf((float)d->head_dim);
   a.max_ctx = max_ctx;
+  a.kv_stable = (d->flags & COSPEC_ATTN_KV_STABLE) ? 1 : 0;
   return from_cuda(launch_verify_attn(a, pl, err, static_cast<cudaStream_t>(stream)));
 }
 

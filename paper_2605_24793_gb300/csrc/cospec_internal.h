@@ -50,6 +50,7 @@ struct AttnArgs {
   int B, R, Hq, Hkv, D, P, max_pages, num_pages;
   float scale;
   int max_ctx;
+  int kv_stable;   // cache-side reads may start before the previous kernel finishes
 };
 struct AttnPlan {
   int mt, wk, nrp;

@@ -37,6 +37,7 @@ struct AttnParams {
   int B, R, Hq, Hkv, G, NR;
   int max_pages, num_pages;
   float scale_log2;
+  int kv_stable;
   int* err;
 };
 
@@ -207,7 +208,14 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
     fence_barrier_init();
   }
   __syncthreads();
-  griddep_wait();                        // inputs may come from the previous kernel
+  // Let the next kernel of the stream start launching right away: its CTAs
+  // take the SMs' free slots and, with the stable-cache promise, stream their
+  // cache tiles while this kernel computes (their own waits keep the order).
+  griddep_launch_dependents();
+  // Without the stable-cache promise, wait for the previous kernel before
+  // reading anything; with it, only q and the block K/V (read below, after
+  // the wait) may come from that kernel, so the cache stream starts now.
+  if (!p.kv_stable) griddep_wait();
 
   const int C = p.ctx_len[b];
   const bool bad = (C < 0) || (C > p.max_pages * PAGE);
@@ -237,6 +245,14 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
       tma_prefetch_desc(&map_vp);
     }
     const uint64_t pol = l2_policy_evict_first();
+    bool waited = !p.kv_stable;
+    if (do_blk && p.R > 0) {
+      // the block K/V is written by the previous kernel: wait first
+      if (!waited) {
+        griddep_wait();
+        waited = true;
+      }
+    }
     if (do_blk && lane == 0) {
       // one box per tensor: KBR rows from block row 0 of this head, both halves
       // (rows past R belong to the next sequence or are zero-filled; masked)
@@ -275,8 +291,10 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
       }
       __syncwarp();
     }
+    if (!waited) griddep_wait();
   } else {
     // ---------------------------------------------------------- consumer warps
+    if (p.kv_stable) griddep_wait();     // q is written by the previous kernel
     // Query fragments (A operand, 16 rows x D) of this warp's row tile.
     uint32_t qf[D / 16][4];
     {
@@ -360,7 +378,6 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
     l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
     l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
   }
-  griddep_launch_dependents();
   __syncthreads();
 
   // CTA partial: rows of every warp, key groups merged (stage ring reused).
@@ -395,29 +412,40 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
       }
     }
     __syncthreads();
-    for (int e = tid; e < NRP * (D / 4); e += NTT) {
-      const int r = e / (D / 4), c = (e % (D / 4)) * 4;
+    // Per row: the common maximum, each key group's weight and the total sum,
+    // computed once (kept in the partial row's (m, l) slots) ...
+    for (int r = tid; r < NRP; r += NTT) {
       const int rt = r / 16, ri = r % 16;
       float M = -INFINITY;
 #pragma unroll
       for (int w = 0; w < WK; ++w) M = fmaxf(M, red[((rt * WK + w) * 16 + ri) * PD + D]);
       float L = 0.f;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (M != -INFINITY) {
 #pragma unroll
-        for (int w = 0; w < WK; ++w) {
-          const float* wr_ = red + ((rt * WK + w) * 16 + ri) * PD;
-          const float sc = exp2_approx(wr_[D] - M);
-          L += wr_[D + 1] * sc;
-          const float4 v = *reinterpret_cast<const float4*>(wr_ + c);
-          acc.x += v.x * sc;
-          acc.y += v.y * sc;
-          acc.z += v.z * sc;
-          acc.w += v.w * sc;
-        }
+      for (int w = 0; w < WK; ++w) {
+        float* wr_ = red + ((rt * WK + w) * 16 + ri) * PD;
+        const float sc = (M == -INFINITY) ? 0.f : exp2_approx(wr_[D] - M);
+        L += wr_[D + 1] * sc;
+        wr_[D + 2] = sc;
+      }
+      *reinterpret_cast<float2*>(part + r * PD + D) = make_float2(M, L);
+    }
+    __syncthreads();
+    // ... then every output chunk is a weighted sum of the key groups' chunks.
+    for (int e = tid; e < NRP * (D / 4); e += NTT) {
+      const int r = e / (D / 4), c = (e % (D / 4)) * 4;
+      const int rt = r / 16, ri = r % 16;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int w = 0; w < WK; ++w) {
+        const float* wr_ = red + ((rt * WK + w) * 16 + ri) * PD;
+        const float sc = wr_[D + 2];
+        const float4 v = *reinterpret_cast<const float4*>(wr_ + c);
+        acc.x += v.x * sc;
+        acc.y += v.y * sc;
+        acc.z += v.z * sc;
+        acc.w += v.w * sc;
       }
       *reinterpret_cast<float4*>(part + r * PD + c) = acc;
-      if (c == 0) *reinterpret_cast<float2*>(part + r * PD + D) = make_float2(M, L);
     }
   }
   fence_proxy_async_smem();              // the bulk copies below read `part`
@@ -609,6 +637,7 @@ cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& pl, int* err,
   p.max_pages = a.max_pages;
   p.num_pages = a.num_pages;
   p.scale_log2 = a.scale * 1.4426950408889634f;
+  p.kv_stable = a.kv_stable;
   p.err = err;
 #define X(DD, MM, WW)                                      \
   if (a.D == DD && pl.mt == MM && pl.wk == WW)             \

@@ -68,8 +68,11 @@ class VerifyRound:
     def attention(self, l: int) -> torch.Tensor:
         pl = 0 if self.k_pages.shape[0] == 1 else l
         out = self.attn_out[l if self.attn_out.shape[0] > 1 else 0]
+        # Layers after the first follow another attention launch, which writes
+        # neither the context lengths, the page table nor the cached pages.
         return C.verify_attn(self.q[l], self.k_blk[l], self.v_blk[l], self.k_pages[pl],
-                             self.v_pages[pl], self.page_table, self.ctx_len, out, self.max_ctx)
+                             self.v_pages[pl], self.page_table, self.ctx_len, out, self.max_ctx,
+                             kv_stable=l > 0)
 
     def lmhead(self):
         return C.lmhead_argmax_features(self.hidden, self.w, self.draft_for_row, self.argmax,

@@ -48,7 +48,7 @@ def test_status_strings(lib):
 
 def _dims(**kw):
     d = dict(batch=2, rows=6, num_q_heads=32, num_kv_heads=8, head_dim=128, page_size=16,
-             max_pages_per_seq=300, num_pages=600, softmax_scale=0.0)
+             max_pages_per_seq=300, num_pages=600, softmax_scale=0.0, flags=0)
     d.update(kw)
     return C.AttnDims(*d.values())
 
