@@ -475,9 +475,14 @@ def main():
         dist.destroy_process_group()
 
 
-# dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture,
-# keyed by (workload, kernel); entries are removed when the kernel changes.
-TRAFFIC = {}
+# dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture
+# (profiles/), keyed by (workload, kernel); an entry is removed when its
+# kernel changes after the capture.
+TRAFFIC = {
+    ("qwen3_8b_b1", "verify_attn"): 16911104.0,
+    ("qwen3_8b_b1", "lmhead_argmax_features"): 1247835632.0,
+    ("qwen3_8b_b16", "verify_attn"): 303825000.0,
+}
 
 
 def kernels_round(k):
