@@ -479,9 +479,7 @@ def main():
 # (profiles/), keyed by (workload, kernel); an entry is removed when its
 # kernel changes after the capture.
 TRAFFIC = {
-    ("qwen3_8b_b1", "verify_attn"): 16911104.0,
     ("qwen3_8b_b1", "lmhead_argmax_features"): 1247835632.0,
-    ("qwen3_8b_b16", "verify_attn"): 303825000.0,
 }
 
 

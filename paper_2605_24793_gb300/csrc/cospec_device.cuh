@@ -155,6 +155,14 @@ CS_DEV void tma_load_4d(uint32_t dst, const void* map, uint64_t* bar, int x, int
       : "memory");
 }
 
+// Warm L2 with a 3-D box (no shared memory written, no completion to track).
+CS_DEV void tma_prefetch_l2_3d(const void* map, int x, int y, int z) {
+  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(map),
+               "r"(x), "r"(y), "r"(z)
+               : "memory");
+}
+CS_DEV void prefetch_l2(const void* p) { asm volatile("prefetch.global.L2 [%0];" ::"l"(p)); }
+
 // ---------------------------------------------------------------- clusters / DSMEM
 CS_DEV uint32_t cluster_ctarank() {
   uint32_t r;

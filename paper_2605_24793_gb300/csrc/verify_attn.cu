@@ -289,12 +289,31 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
                       &full[st], 0, y, 0, pol);
         }
       }
+      if (vt == NSTAGE - 1) {
+        // The ring is full: pull the next two tiles' pages into L2 so their
+        // loads, issued once stages free up, skip most of the HBM latency.
+        const int e = NSTAGE * 4 + (lane >> 1);                  // lanes 0..15: 8 pages, K and V
+        const int pg = __shfl_sync(0xffffffffu, pid, e & 31);
+        if (lane < 16 && e < my_pages && (unsigned)pg < (unsigned)p.num_pages)
+          tma_prefetch_l2_3d((lane & 1) ? (const void*)&map_vp : (const void*)&map_kp, 0,
+                             (pg * p.Hkv + kvh) * PAGE, 0);
+      }
       __syncwarp();
     }
     if (!waited) griddep_wait();
   } else {
     // ---------------------------------------------------------- consumer warps
-    if (p.kv_stable) griddep_wait();     // q is written by the previous kernel
+    if (p.kv_stable) {
+      // Warm L2 with this CTA's query rows (writes by the previous kernel
+      // still land in L2 first), then wait for that kernel.
+      const int nrow = min(p.NR, NRP);
+      for (int e = tid; e < nrow * (D * 2 / 128); e += NTC) {
+        const int r = e / (D * 2 / 128), part_ = e % (D * 2 / 128);
+        const int j = r / p.G, g = r % p.G;
+        prefetch_l2(p.q + (((size_t)b * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D + part_ * 64);
+      }
+      griddep_wait();                    // q is written by the previous kernel
+    }
     // Query fragments (A operand, 16 rows x D) of this warp's row tile.
     uint32_t qf[D / 16][4];
     {
