@@ -600,11 +600,14 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
   pl.mt = variant_mt(NR);
   pl.wk = (pl.mt >= 4) ? 1 : 4 / pl.mt;
   pl.nrp = pl.mt * 16;
-  // Split each (sequence, head) over a cluster of S CTAs: enough CTAs for
-  // about four per SM over the launch, at least 4 cache tiles per CTA.
+  // Split each (sequence, head) over a cluster of S CTAs: about one wave at
+  // two CTAs per SM, no CTA with more than 256 cache tiles (long contexts),
+  // at least 4 tiles per CTA, at most 16 CTAs per cluster.
   const int tiles = (max_ctx + KT - 1) / KT;
   const long long units = (long long)B * Hkv;
-  const long long want = (4LL * num_sms + units - 1) / (units > 0 ? units : 1);
+  const long long want_wave = (2LL * num_sms + units - 1) / (units > 0 ? units : 1);
+  const long long want_len = (tiles + 255) / 256;
+  const long long want = want_wave > want_len ? want_wave : want_len;
   int S = 1;
   while (S < 16 && S < want && (S * 2) * 4 <= tiles) S *= 2;
   if (pl.mt == 8) S = 1;   // the 128-row partials leave no room to receive a cluster's pushes
