@@ -291,9 +291,8 @@ def main():
             args.steps = 10
         return run_reference(args)
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    from paper_2605_24793_gb300 import replicas
+    world, rank, local_rank = replicas.env_ranks()
     torch.cuda.set_device(local_rank)
     dist = None
     if world > 1:
@@ -382,12 +381,9 @@ def main():
     attn_ms = float(np.mean([ev[k][0].elapsed_time(ev[k][1]) for k in range(K)]))
     lm_ms = float(np.mean([ev[k][1].elapsed_time(ev[k][2]) for k in range(K)]))
     tail_ms = float(np.mean([ev[k][2].elapsed_time(ev[k][3]) for k in range(K)]))
-    if dist:
-        t = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = replicas.max_over_ranks(total_ms, dist, torch.device("cuda", local_rank))
     ms_per_step = total_ms / K
-    value = world * cfg.batch * cfg.rows / (ms_per_step * 1e-3)
+    value = replicas.job_throughput(cfg.batch * cfg.rows, ms_per_step * 1e-3, world)
     if C.get_device_error(stream) != 0:
         raise RuntimeError("device error word set during the timed region")
     s_mean = float(rnd.accept_len.float().mean().item())
@@ -518,10 +514,8 @@ def end_to_end(cfg, rnd, step, stream, steps, dist):
     for _ in range(steps):
         e2e_step()
     dt = time.perf_counter() - t0
-    if dist:
-        t = torch.tensor([dt], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        dt = float(t.item())
+    from paper_2605_24793_gb300 import replicas
+    dt = replicas.max_over_ranks(dt, dist, torch.device("cuda", torch.cuda.current_device()))
     return {"per_rank_value": cfg.batch * cfg.rows * steps / dt, "unit": UNIT,
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "ms_per_step": 1e3 * dt / steps, "steps": steps,
