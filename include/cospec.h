@@ -101,7 +101,7 @@ COSPEC_API int cospec_num_sms(void);
  *    CTAs of one thread-block cluster, whose partial results merge in
  *    distributed shared memory.
  *    Supported: head_dim in {64, 128}; page_size == 16; rows <= 32;
- *    num_q_heads % num_kv_heads == 0; (num_q_heads / num_kv_heads) * rows <= 128.
+ *    num_q_heads % num_kv_heads == 0; (num_q_heads / num_kv_heads) * rows <= 512.
  * ------------------------------------------------------------------------ */
 typedef struct {
   int batch;

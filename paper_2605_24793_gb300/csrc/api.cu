@@ -134,7 +134,7 @@ static int check_attn_dims(const cospec_attn_dims* d) {
   if (d->head_dim != 64 && d->head_dim != 128) return COSPEC_ERR_UNSUPPORTED;
   if (d->page_size != 16) return COSPEC_ERR_UNSUPPORTED;
   if (d->rows > 32) return COSPEC_ERR_UNSUPPORTED;
-  if ((d->num_q_heads / d->num_kv_heads) * d->rows > 128) return COSPEC_ERR_UNSUPPORTED;
+  if ((d->num_q_heads / d->num_kv_heads) * d->rows > 512) return COSPEC_ERR_UNSUPPORTED;
   return COSPEC_OK;
 }
 

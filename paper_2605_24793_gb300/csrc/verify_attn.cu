@@ -34,7 +34,9 @@ struct AttnParams {
   const int32_t* page_table;
   const int32_t* ctx_len;
   __nv_bfloat16* out;
-  int B, R, Hq, Hkv, G, NR;
+  int B, R, Hq, Hkv, G;
+  int NRT;         // query rows of a (sequence, KV head): G * R
+  int RG;          // row groups of at most 64 rows per (sequence, KV head)
   int max_pages, num_pages;
   float scale_log2;
   int kv_stable;
@@ -195,7 +197,9 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
 
   const int S = (int)cluster_nctarank();
   const int rank = (int)cluster_ctarank();
-  const int kvh = blockIdx.y, b = blockIdx.z;
+  const int kvh = blockIdx.y / p.RG, rg = blockIdx.y % p.RG, b = blockIdx.z;
+  const int row_g0 = rg * 64;                      // first query row of this group
+  const int NR = min(64, p.NRT - row_g0);          // rows of this group (<= NRP)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
   if (tid == 0) {
@@ -306,9 +310,8 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
     if (p.kv_stable) {
       // Warm L2 with this CTA's query rows (writes by the previous kernel
       // still land in L2 first), then wait for that kernel.
-      const int nrow = min(p.NR, NRP);
-      for (int e = tid; e < nrow * (D * 2 / 128); e += NTC) {
-        const int r = e / (D * 2 / 128), part_ = e % (D * 2 / 128);
+      for (int e = tid; e < NR * (D * 2 / 128); e += NTC) {
+        const int r = row_g0 + e / (D * 2 / 128), part_ = e % (D * 2 / 128);
         const int j = r / p.G, g = r % p.G;
         prefetch_l2(p.q + (((size_t)b * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D + part_ * 64);
       }
@@ -318,8 +321,8 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
     uint32_t qf[D / 16][4];
     {
       auto row_ptr = [&](int r) -> const __nv_bfloat16* {
-        if (r >= p.NR) return nullptr;
-        const int j = r / p.G, g = r % p.G;
+        if (r >= NR) return nullptr;
+        const int j = (row_g0 + r) / p.G, g = (row_g0 + r) % p.G;
         return p.q + (((size_t)b * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D;
       };
       const __nv_bfloat16* q0 = row_ptr(r0);
@@ -333,7 +336,7 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
         qf[kk][3] = q1 ? __ldg(reinterpret_cast<const uint32_t*>(q1 + col + 8)) : 0u;
       }
     }
-    const int j0 = min(r0 / p.G, p.R - 1), j1 = min(r1 / p.G, p.R - 1);
+    const int j0 = min((row_g0 + r0) / p.G, p.R - 1), j1 = min((row_g0 + r1) / p.G, p.R - 1);
 #pragma unroll
     for (int i = 0; i < D / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
 
@@ -474,7 +477,7 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
   // Each CTA sends its partial rows to their owners with one bulk shared-
   // to-shared copy per owner (thread-level remote accesses are slow); the
   // owner merges the S received copies from its own shared memory.
-  const int rpo = (p.NR + S - 1) / S;
+  const int rpo = (NR + S - 1) / S;
   const float* src = part;
   if (S > 1) {
     if (tid == 0) mbar_arrive_expect_tx(recv_bar, (uint32_t)(S * rpo * LY::ROWP));
@@ -494,7 +497,7 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
   for (int e = tid; e < rpo * (D / 4); e += NTT) {
     const int rr = e / (D / 4), c = (e % (D / 4)) * 4;
     const int r = row0 + rr;
-    if (r >= p.NR) break;
+    if (r >= NR) break;
     float M = -INFINITY;
     for (int s2 = 0; s2 < S; ++s2) M = fmaxf(M, src[(s2 * rpo + rr) * PD + D]);
     float L = 0.f;
@@ -512,7 +515,7 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
       }
     }
     const float inv = (L > 0.f) ? 1.f / L : 0.f;
-    const int j = r / p.G, g = r % p.G;
+    const int j = (row_g0 + r) / p.G, g = (row_g0 + r) % p.G;
     __nv_bfloat16* dst = p.out + (((size_t)b * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D + c;
     uint2 pk;
     pk.x = pack_bf16(acc.x * inv, acc.y * inv);
@@ -541,7 +544,7 @@ cudaError_t launch_t(const CUtensorMap* maps, const AttnParams& p, int S, int B,
     configured[dev] = true;
   }
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(S, Hkv, B);
+  cfg.gridDim = dim3(S, Hkv * p.RG, B);
   cfg.blockDim = dim3(MT * WK * 32 + 32, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
@@ -582,21 +585,22 @@ int max_cluster_t(int S, int Hkv, int B) {
   return n;
 }
 
-int variant_mt(int NR) {
+int variant_mt(int NR) {   // NR <= 64
   if (NR <= 16) return 1;
   if (NR <= 32) return 2;
-  if (NR <= 64) return 4;
-  return 8;
+  return 4;
 }
 
 #define COSPEC_ATTN_VARIANTS(X) \
-  X(128, 1, 4) X(128, 2, 2) X(128, 4, 1) X(128, 8, 1) X(64, 1, 4) X(64, 2, 2) X(64, 4, 1) X(64, 8, 1)
+  X(128, 1, 4) X(128, 2, 2) X(128, 4, 1) X(64, 1, 4) X(64, 2, 2) X(64, 4, 1)
 
 }  // namespace
 
 AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int num_sms) {
   AttnPlan pl{};
-  const int NR = (Hq / Hkv) * R;
+  const int NRT = (Hq / Hkv) * R;
+  const int RG = (NRT + 63) / 64;                  // row groups of at most 64 rows
+  const int NR = NRT < 64 ? NRT : 64;
   pl.mt = variant_mt(NR);
   pl.wk = (pl.mt >= 4) ? 1 : 4 / pl.mt;
   pl.nrp = pl.mt * 16;
@@ -604,13 +608,12 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
   // two CTAs per SM, no CTA with more than 256 cache tiles (long contexts),
   // at least 4 tiles per CTA, at most 16 CTAs per cluster.
   const int tiles = (max_ctx + KT - 1) / KT;
-  const long long units = (long long)B * Hkv;
+  const long long units = (long long)B * Hkv * RG;
   const long long want_wave = (2LL * num_sms + units - 1) / (units > 0 ? units : 1);
   const long long want_len = (tiles + 255) / 256;
   const long long want = want_wave > want_len ? want_wave : want_len;
   int S = 1;
   while (S < 16 && S < want && (S * 2) * 4 <= tiles) S *= 2;
-  if (pl.mt == 8) S = 1;   // the 128-row partials leave no room to receive a cluster's pushes
   pl.cluster = S;
   pl.tiles_per_split = (tiles + S - 1) / S;
   pl.max_splits = S;
@@ -655,7 +658,8 @@ cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& pl, int* err,
   p.Hq = a.Hq;
   p.Hkv = a.Hkv;
   p.G = a.Hq / a.Hkv;
-  p.NR = p.G * a.R;
+  p.NRT = p.G * a.R;
+  p.RG = (p.NRT + 63) / 64;
   p.max_pages = a.max_pages;
   p.num_pages = a.num_pages;
   p.scale_log2 = a.scale * 1.4426950408889634f;

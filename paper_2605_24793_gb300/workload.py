@@ -243,7 +243,7 @@ def make_round_inputs(cfg: RoundConfig, device="cpu", extra_tokens: int = 0,
     return out
 
 
-def synth_drafts(cfg: RoundConfig, ranked_ids: np.ndarray) -> np.ndarray:
+def synth_drafts(cfg: RoundConfig, ranked_ids: np.ndarray, round_index: int = 0) -> np.ndarray:
     """Draft block y_hat [B, K] for a chain draft.
 
     ``ranked_ids`` [B, R, t] are, per block row, the target's top-t token ids
@@ -251,8 +251,10 @@ def synth_drafts(cfg: RoundConfig, ranked_ids: np.ndarray) -> np.ndarray:
     checked against row i-1.  With probability 1 - mismatch_rate the draft is
     the rank-1 id; otherwise it is drawn uniformly from ranks 2..topk
     (``mismatch_topk`` > 1) or from all other ids (``mismatch_topk`` == 0).
+    ``round_index`` selects an independent draw for each round of a
+    multi-round run.
     """
-    rng = np.random.default_rng(seed_of(cfg, "drafts"))
+    rng = np.random.default_rng(seed_of(cfg, "drafts") + 7919 * round_index)
     B, K = cfg.batch, cfg.k
     draft = np.empty((B, K), dtype=np.int32)
     for b in range(B):

@@ -64,6 +64,8 @@ ATTN_CASES = [
     (2, 8, 128, 8, 64, [31, 700], False),           # G = 16 -> 128 rows at head_dim 64
     (2, 1, 32, 8, 128, [0, 1], False),              # K = 0: one row per sequence
     (5, 4, 32, 8, 128, [8191, 40, 63, 64, 2049], True),
+    (1, 26, 32, 8, 128, [4096], False),             # K = 25 (the paper's default): 104 rows, 2 groups
+    (2, 32, 128, 8, 64, [300, 1500], True),         # 512 rows per KV head: 8 row groups
 ]
 
 
