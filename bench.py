@@ -283,6 +283,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--layers", type=int, default=None, help="override the layer count")
+    ap.add_argument("--temperature", type=float, default=None,
+                    help="stochastic decoding: sample the target candidates at this temperature")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -309,7 +311,9 @@ def main():
         cfg = cfg.replace(layers=args.layers)
     inp = W.make_round_inputs(cfg, device="cuda")
     draft = gpu_drafts(cfg, inp)
-    rnd = VerifyRound(inp, draft, cfg.lam)
+    rnd = VerifyRound(inp, draft, cfg.lam, temperature=args.temperature,
+                      seed=W.sample_seed(cfg))
+    lm_name = "lmhead_argmax_features" if args.temperature is None else "lmhead_sample_features"
     stream = torch.cuda.Stream()
     torch.cuda.synchronize()
 
@@ -404,7 +408,7 @@ def main():
                         "gbs": a_bytes / (attn_launch_ms * 1e-3) / 1e9,
                         "frac_hbm": a_bytes / (attn_launch_ms * 1e-3) / 1e9 / hbm,
                         "share": attn_ms / (attn_ms + lm_ms + tail_ms)},
-        "lmhead_argmax_features": {"ms_per_launch": lm_ms, "bytes_per_launch": lm_bytes,
+        lm_name: {"ms_per_launch": lm_ms, "bytes_per_launch": lm_bytes,
                                    "flops_per_launch": lmhead_flops(cfg),
                                    "gbs": lm_bytes / (lm_ms * 1e-3) / 1e9,
                                    "tflops": lmhead_flops(cfg) / (lm_ms * 1e-3) / 1e12,
@@ -420,12 +424,12 @@ def main():
         roof = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                 "frac": achieved / hbm, "traffic": None}
     elif lm_t_hbm >= lm_t_tc:
-        dom = "lmhead_argmax_features"
+        dom = lm_name
         achieved = lm_bytes / (lm_ms * 1e-3) / 1e9
         roof = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                 "frac": achieved / hbm, "traffic": None}
     else:
-        dom = "lmhead_argmax_features"
+        dom = lm_name
         achieved = lmhead_flops(cfg) / (lm_ms * 1e-3) / 1e12
         roof = {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": tflops_peak,
                 "unit": "TFLOP/s", "frac": achieved / tflops_peak, "traffic": None}
@@ -456,6 +460,8 @@ def main():
                        "q_heads": cfg.q_heads, "kv_heads": cfg.kv_heads,
                        "head_dim": cfg.head_dim, "hidden": cfg.hidden, "vocab": cfg.vocab,
                        "page_size": cfg.page_size, "lambda": cfg.lam,
+                       "decoding": ("greedy" if args.temperature is None
+                                    else f"sampled, T={args.temperature}"),
                        "parallelism": f"replicas x{world}",
                        "l2": (f"inputs larger than L2: {(a_bytes * cfg.layers + lm_bytes) / 1e9:.2f}"
                               " GB streamed per step vs 129 MB L2"),

@@ -155,6 +155,33 @@ COSPEC_API int cospec_lmhead_argmax_features(int M, int d, int V, const uint16_t
                                              int32_t* argmax, float* stats, void* ws,
                                              size_t ws_bytes, void* stream);
 
+/* Stochastic decoding (Sec. 3.1 "Stochastic decoding"; App. C.3 draws the
+ * draft and target candidates at temperature T = 1 and arbitrates between
+ * the pair exactly as in greedy decoding).  Same contraction, statistics and
+ * workspace as cospec_lmhead_argmax_features, but the target candidate
+ * written to sample[m] is a draw from softmax(x / T) instead of the argmax:
+ *
+ *   sample[m] = argmax_v ( x_v / T + g_{m,v} ),  g = -log(-log u)   (Gumbel-max)
+ *   u_{m,v}   = (floor(r / 2^9) + 0.5) / 2^23,  r = output (m mod 4) of
+ *               Philox4x32-10 at counter (v, floor(m / 4), 0, 0) under the
+ *               key (seed mod 2^32, floor(seed / 2^32))
+ *
+ * (Salmon et al., SC 2011), ties going to the lowest id.  stats[m][*] are
+ * the statistics of the logits x themselves, as in the greedy call.
+ *
+ *    temperature > 0 and finite (1 for the paper's stochastic setting).
+ *    seed      DEVICE pointer to one uint64 (8-byte aligned), read when the
+ *              kernel runs, so a captured graph draws fresh noise whenever
+ *              the caller rewrites it between replays.
+ *    sample    int32 [M];  other arguments as for the greedy call.
+ * This is not distribution-preserving speculative sampling: the paper's
+ * method uses the sampled pair as two candidates for arbitration. */
+COSPEC_API int cospec_lmhead_sample_features(int M, int d, int V, const uint16_t* hidden,
+                                             const uint16_t* w, const int32_t* draft_for_row,
+                                             float temperature, const uint64_t* seed,
+                                             int32_t* sample, float* stats, void* ws,
+                                             size_t ws_bytes, void* stream);
+
 /* Same computation and outputs as cospec_lmhead_argmax_features, for callers
  * that cannot allocate device memory or hand this library a workspace -- for
  * example a serving engine that reserves nearly all HBM for its KV cache and

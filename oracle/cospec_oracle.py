@@ -15,6 +15,10 @@ Pins (what fixes each function other than itself; see tests/test_oracle_*.py):
                         head mapping, causality, paged == contiguous.
   lmhead_stats          closed forms (one-hot logits, uniform logits, two
                         classes), tie-break, torch float64 cross-check.
+  row_stats_sampled     Philox4x32-10 known-answer vectors of the generator's
+                        authors; Gumbel moments (Euler's constant, pi^2/6);
+                        sample frequencies against softmax; T -> 0 gives the
+                        argmax.
   arbitration_features  hand-derived golden case (tests/golden).
   arbitration_mlp       parity unpinned: the paper defines no feature MLP;
                         only a hand-computed 2-input example fixes the formula.
@@ -148,6 +152,30 @@ def row_stats(x: np.ndarray, draft_for_row) -> tuple:
     draft_logit = np.where(d >= 0, x[rows, np.clip(d, 0, V - 1)], np.nan)
     stats = np.stack([mx, second, lse, entropy, draft_logit], axis=1)
     return am.astype(np.int64), stats
+
+
+def gumbel_keys(x: np.ndarray, seed: int, temperature: float = 1.0) -> np.ndarray:
+    """Perturbed keys x_v / T + g_v of the Gumbel-max rule, g = -log(-log u) with
+    u from the Philox4x32-10 stream of `seed` (oracle/philox.py), [M, V]."""
+    from .philox import gumbel_noise
+    x = np.asarray(x, dtype=F64)
+    return x / temperature + gumbel_noise(seed, x.shape[0], x.shape[1])
+
+
+def row_stats_sampled(x: np.ndarray, draft_for_row, seed: int, temperature: float = 1.0):
+    """Stochastic decoding (Sec. 3.1 "Stochastic decoding", App. C.3): the
+    target candidate is a sample of softmax(x / T), drawn as the argmax of the
+    Gumbel-perturbed keys (lowest id among exact ties).  The statistics are
+    those of the logits themselves (as in row_stats).
+    Returns (sample int64 [M], stats float64 [M, 5])."""
+    _, stats = row_stats(x, draft_for_row)
+    return np.argmax(gumbel_keys(x, seed, temperature), axis=1).astype(np.int64), stats
+
+
+def lmhead_stats_sampled(hidden, w, draft_for_row, seed: int, temperature: float = 1.0,
+                         vocab_chunk: int = 16384):
+    """LM-head contraction with a temperature-T sample in place of the argmax."""
+    return row_stats_sampled(lmhead_logits(hidden, w, vocab_chunk), draft_for_row, seed, temperature)
 
 
 def lmhead_stats(hidden, w, draft_for_row, vocab_chunk: int = 16384):
@@ -329,11 +357,15 @@ def commit_kv(k_blk, v_blk, k_pages, v_pages, page_table, ctx_len, s, page_size:
 # ---------------------------------------------------------------------------
 
 def cospec_round(inp: dict, draft, lam: float, mode: int = POLICY_MLP,
-                 with_attention: bool = True, with_commit: bool = True) -> dict:
+                 with_attention: bool = True, with_commit: bool = True,
+                 sample_seed: Optional[int] = None, temperature: float = 1.0) -> dict:
     """All five steps on the inputs drawn by the workload generator.
 
     ``inp`` holds q, k_blk, v_blk, k_pages, v_pages (per layer, leading L),
-    page_table_np, ctx_len_np, hidden, w, mlp, cfg.
+    page_table_np, ctx_len_np, hidden, w, mlp, cfg.  With ``sample_seed`` the
+    target candidates are temperature samples (stochastic decoding, Sec. 3.1)
+    instead of the argmax; ``key_margin`` [B, R] is the gap between the two
+    largest keys that decided each row's candidate (logit or perturbed key).
     """
     cfg = inp["cfg"]
     B, K, R = cfg.batch, cfg.k, cfg.rows
@@ -348,7 +380,15 @@ def cospec_round(inp: dict, draft, lam: float, mode: int = POLICY_MLP,
     dfr = np.full((B, R), -1, dtype=np.int64)
     dfr[:, :K] = d
     x = lmhead_logits(inp["hidden"], inp["w"])
-    am, st = row_stats(x, dfr.reshape(-1))
+    if sample_seed is None:
+        am, st = row_stats(x, dfr.reshape(-1))
+        keys = x
+    else:
+        am, st = row_stats_sampled(x, dfr.reshape(-1), sample_seed, temperature)
+        keys = gumbel_keys(x, sample_seed, temperature)
+    top2 = np.sort(keys, axis=1)[:, -2:] if keys.shape[1] > 1 else np.concatenate(
+        [np.full((keys.shape[0], 1), -np.inf), keys], axis=1)
+    out["key_margin"] = (top2[:, 1] - top2[:, 0]).reshape(B, R)
     out["logits"] = x
     out["argmax"] = am.reshape(B, R)
     out["stats"] = st.reshape(B, R, 5)

@@ -21,7 +21,8 @@ DEVERR_PAGE, DEVERR_CTX, DEVERR_TOKEN, DEVERR_TIMEOUT = 1, 2, 4, 8
 
 EXPORTED = ("cospec_status_string", "cospec_get_device_error", "cospec_num_sms",
             "cospec_verify_attn", "cospec_lmhead_workspace", "cospec_lmhead_argmax_features",
-            "cospec_arbitrate", "cospec_accept_commit", "cospec_lmhead_argmax_features_noalloc")
+            "cospec_arbitrate", "cospec_accept_commit", "cospec_lmhead_argmax_features_noalloc",
+            "cospec_lmhead_sample_features")
 
 
 class AttnDims(ctypes.Structure):
@@ -61,6 +62,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "cospec_lmhead_workspace": (_sz, [_i, _i, _i]),
         "cospec_lmhead_argmax_features": (_i, [_i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
         "cospec_lmhead_argmax_features_noalloc": (_i, [_i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp]),
+        "cospec_lmhead_sample_features": (_i, [_i, _i, _i, _vp, _vp, _vp, _f, _vp, _vp, _vp, _vp,
+                                               _sz, _vp]),
         "cospec_arbitrate": (_i, [_i, _i, _vp, _vp, _vp, _i, _vp, _vp, _vp, _f, _f, _i, _vp, _vp, _vp]),
         "cospec_accept_commit": (_i, [_i, _i, _i, _PDIMS, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                       ctypes.c_longlong, _vp, _vp, _vp, _vp, _vp]),
@@ -160,6 +163,31 @@ def lmhead_argmax_features(hidden, w, draft_for_row, argmax, stats, ws, stream=N
         M, d, V, _ptr(hidden), _ptr(w), _ptr(draft_for_row), _ptr(argmax), _ptr(stats), _ptr(ws),
         ws.numel(), _stream(stream)))
     return argmax, stats
+
+
+def lmhead_sample_features(hidden, w, draft_for_row, temperature: float, seed, sample, stats, ws,
+                           stream=None):
+    """Stochastic-decoding LM head (Sec. 3.1, App. C.3): sample [M] is a
+    Gumbel-max draw from softmax(x / T) with Philox4x32-10 noise keyed by the
+    int64 device scalar ``seed`` (read when the kernel runs); stats as in
+    lmhead_argmax_features."""
+    _req(hidden, torch.bfloat16, "hidden", 2)
+    _req(w, torch.bfloat16, "w", 2)
+    _req(draft_for_row, torch.int32, "draft_for_row", 1)
+    _req(sample, torch.int32, "sample", 1)
+    _req(stats, torch.float32, "stats", 2)
+    _req(ws, torch.uint8, "ws", 1)
+    _req(seed, torch.int64, "seed")
+    if seed.numel() != 1:
+        raise ValueError("seed must hold one value")
+    M, d = hidden.shape
+    V = w.shape[0]
+    if w.shape[1] != d or draft_for_row.numel() != M or sample.numel() != M or tuple(stats.shape) != (M, 5):
+        raise ValueError("inconsistent LM-head shapes")
+    _check(load_library().cospec_lmhead_sample_features(
+        M, d, V, _ptr(hidden), _ptr(w), _ptr(draft_for_row), float(temperature), _ptr(seed),
+        _ptr(sample), _ptr(stats), _ptr(ws), ws.numel(), _stream(stream)))
+    return sample, stats
 
 
 def lmhead_argmax_features_noalloc(hidden, w, draft_for_row, argmax, stats, stream=None):

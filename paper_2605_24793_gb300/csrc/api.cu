@@ -227,6 +227,32 @@ COSPEC_API int cospec_lmhead_argmax_features(int M, int d, int V, const uint16_t
                                  stats, ws, pl, err, static_cast<cudaStream_t>(stream)));
 }
 
+COSPEC_API int cospec_lmhead_sample_features(int M, int d, int V, const uint16_t* hidden,
+                                             const uint16_t* w, const int32_t* draft_for_row,
+                                             float temperature, const uint64_t* seed,
+                                             int32_t* sample, float* stats, void* ws,
+                                             size_t ws_bytes, void* stream) {
+  CS_CHECK_ARG(M >= 0 && d > 0 && V > 0);
+  CS_CHECK_ARG(temperature > 0.f && isfinite(temperature) && isfinite(1.0f / temperature));
+  if (M == 0) return COSPEC_OK;
+  CS_CHECK_ARG(hidden && w && draft_for_row && sample && stats && seed);
+  CS_CHECK_ARG((reinterpret_cast<uintptr_t>(seed) & 7u) == 0);
+  if (d % 64 != 0) return COSPEC_ERR_UNSUPPORTED;
+  if ((long long)V > 0x7fffff00LL) return COSPEC_ERR_UNSUPPORTED;
+  CS_CHECK_ARG(aligned16(hidden) && aligned16(w));
+  const int sms = device_num_sms();
+  if (sms <= 0) return COSPEC_ERR_CUDA;
+  const LmheadPlan pl = plan_lmhead(M, d, V, sms);
+  if (!ws || ws_bytes < pl.ws_bytes || !aligned16(ws)) return COSPEC_ERR_WORKSPACE;
+  int* err = device_error_word();
+  if (!err) return COSPEC_ERR_CUDA;
+  return from_cuda(launch_lmhead(M, d, V, reinterpret_cast<const __nv_bfloat16*>(hidden),
+                                 reinterpret_cast<const __nv_bfloat16*>(w), draft_for_row, sample,
+                                 stats, ws, pl, err, static_cast<cudaStream_t>(stream),
+                                 reinterpret_cast<const unsigned long long*>(seed),
+                                 1.0f / temperature));
+}
+
 // ---------------------------------------------------------------- arbitration
 COSPEC_API int cospec_arbitrate(int B, int K, const int32_t* draft, const int32_t* argmax,
                                 const float* stats, int mlp_hidden, const float* w1,

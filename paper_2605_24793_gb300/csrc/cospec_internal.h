@@ -77,7 +77,8 @@ LmheadPlan plan_lmhead(int M, int d, int V, int num_sms);
 cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
                           const __nv_bfloat16* w, const int32_t* draft_for_row, int32_t* argmax,
                           float* stats, void* ws, const LmheadPlan& plan, int* err,
-                          cudaStream_t stream);
+                          cudaStream_t stream, const unsigned long long* seed = nullptr,
+                          float inv_temp = 1.f);
 
 // ---------------------------------------------------------------- arbitration
 cudaError_t launch_arbitrate(int B, int K, const int32_t* draft, const int32_t* argmax,

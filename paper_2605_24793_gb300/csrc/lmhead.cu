@@ -8,14 +8,26 @@
 // large operand -- is streamed from HBM exactly once.  Persistent CTAs (one
 // per SM) walk vocabulary tiles; warp 0 issues TMA loads (128B swizzle, W
 // with evict-first, hidden rows with evict-last) into a ring of stages,
-// warp 1 issues tcgen05.mma into one of two TMEM accumulators, warps 2-5 read
+// warp 1 issues tcgen05.mma into one of two TMEM accumulators, warps 2-9 read
 // the finished accumulator with tcgen05.ld and fold it into per-row running
-// statistics while the next tile is multiplied.  A second small kernel
+// statistics while the next tile is multiplied.  A warp may only read the
+// TMEM lane quarter (warp id mod 4), so two epilogue warps share each quarter
+// (128 vocabulary rows / 4) and take alternate 16-column chunks; two warps per
+// SM sub-partition hide each other's shuffle and MUFU latency.  A second small kernel
 // merges the per-CTA partials.
 //
 // Statistics are kept as a tuple (m, i, sec, s, t): max logit, its lowest
 // id, second largest logit, s = sum e^(x-m), t = sum e^(x-m) (x-m); then
 // lse = m + log s and entropy = log s - t/s.
+//
+// Stochastic decoding (Sec. 3.1, App. C.3: candidates drawn at temperature
+// T = 1) uses the same kernel with KEYED = true: the target candidate is a
+// sample of softmax(x / T) taken by the Gumbel-max rule, argmax_v of
+// k_v = x_v / T + g_v with g_v = -log(-log u_v).  u comes from Philox4x32-10
+// (Salmon et al., SC 2011) keyed by a 64-bit seed read from device memory, at
+// counter (v, m / 4, 0, 0), output m % 4, so a thread that owns vocab id v and
+// four consecutive rows makes one generator call.  The tuple then carries the
+// best key k and i becomes its id; m, sec, s, t stay statistics of the logits.
 #include <cuda.h>
 #include <math.h>
 
@@ -30,8 +42,9 @@ namespace {
 constexpr int BM = 128;                 // vocab rows per tile (MMA M)
 constexpr int BK = 64;                  // K elements per stage (one 128-byte swizzle row)
 constexpr int A_BYTES = BM * BK * 2;    // 16 KB
-constexpr int NUM_THREADS = 192;        // TMA warp, MMA warp, 4 epilogue warps
-constexpr int EPI_THREADS = 128;
+constexpr int EPI_WARPS = 8;            // two per TMEM lane quarter
+constexpr int EPI_THREADS = 32 * EPI_WARPS;
+constexpr int NUM_THREADS = 64 + EPI_THREADS;   // TMA warp, MMA warp, epilogue warps
 constexpr int MAX_ROWS = 256;           // rows per pass
 constexpr uint64_t WAIT_NS = 2000000000ull;
 
@@ -41,17 +54,28 @@ struct Stat {
   float sec;
   float s;
   float t;
+  float k;    // KEYED only: largest perturbed key, whose id is i
 };
 
-CS_DEV Stat stat_identity() { return Stat{-INFINITY, 0x7fffffff, -INFINITY, 0.f, 0.f}; }
+CS_DEV Stat stat_identity() { return Stat{-INFINITY, 0x7fffffff, -INFINITY, 0.f, 0.f, -INFINITY}; }
 
+template <bool KEYED>
 CS_DEV Stat stat_merge(const Stat& a, const Stat& b) {
-  const bool a_hi = (a.m > b.m) || (a.m == b.m && a.i < b.i);
+  Stat r;
+  bool a_hi;
+  if (KEYED) {
+    const bool a_key = (a.k > b.k) || (a.k == b.k && a.i < b.i);
+    r.k = a_key ? a.k : b.k;
+    r.i = a_key ? a.i : b.i;
+    a_hi = a.m >= b.m;
+  } else {
+    a_hi = (a.m > b.m) || (a.m == b.m && a.i < b.i);
+    r.i = a_hi ? a.i : b.i;
+    r.k = 0.f;
+  }
   const Stat& hi = a_hi ? a : b;
   const Stat& lo = a_hi ? b : a;
-  Stat r;
   r.m = hi.m;
-  r.i = hi.i;
   r.sec = fmaxf(fmaxf(hi.sec, lo.sec), lo.m);
   if (lo.s > 0.f) {
     const float dm = lo.m - hi.m;
@@ -65,6 +89,7 @@ CS_DEV Stat stat_merge(const Stat& a, const Stat& b) {
   return r;
 }
 
+template <bool KEYED>
 CS_DEV Stat stat_shfl_xor(const Stat& a, int off) {
   Stat r;
   r.m = __shfl_xor_sync(0xffffffffu, a.m, off);
@@ -72,18 +97,52 @@ CS_DEV Stat stat_shfl_xor(const Stat& a, int off) {
   r.sec = __shfl_xor_sync(0xffffffffu, a.sec, off);
   r.s = __shfl_xor_sync(0xffffffffu, a.s, off);
   r.t = __shfl_xor_sync(0xffffffffu, a.t, off);
+  r.k = KEYED ? __shfl_xor_sync(0xffffffffu, a.k, off) : 0.f;
   return r;
 }
 
-CS_DEV Stat stat_of(float x, int v) {
-  return Stat{x, v, -INFINITY, (x == -INFINITY) ? 0.f : 1.f, 0.f};
+CS_DEV Stat stat_of(float x, float k, int v) {
+  return Stat{x, v, -INFINITY, (x == -INFINITY) ? 0.f : 1.f, 0.f, k};
+}
+
+// Philox4x32-10: ten rounds of two 32x32 -> 64-bit products by the
+// multipliers 0xD2511F53 / 0xCD9E8D57, the key advanced by the Weyl
+// increments 0x9E3779B9 / 0xBB67AE85 between rounds.
+CS_DEV uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r) {
+      k0 += 0x9E3779B9u;
+      k1 += 0xBB67AE85u;
+    }
+    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+  }
+  return c;
+}
+
+// Standard Gumbel variate g = -log(E), E = -log(u) ~ Exp(1), from 32 random
+// bits: u = (floor(r / 2^9) + 0.5) / 2^23 is an odd multiple of 2^-24 in (0, 1),
+// exact in float32, and so is w = 1 - u.  Near u = 1 (w < 1/64) E comes from
+// the series -log(1 - w) = w + w^2/2 + w^3/3 + w^4/4 + ..., whose truncation
+// is below 1e-8 relative there; elsewhere |log u| > 1/64 and the fast
+// logarithm's absolute error (about 4e-7) is at most ~3e-5 relative.  The
+// largest keys, which decide the sample, come from the series branch.
+CS_DEV float gumbel_of(uint32_t r) {
+  const float u = ((float)(r >> 9) + 0.5f) * 1.1920928955078125e-7f;
+  const float w = 1.f - u;
+  const float e_series = w * fmaf(w, fmaf(w, fmaf(w, 0.25f, 0.333333343f), 0.5f), 1.f);
+  const float e = (w < 0.015625f) ? e_series : -__logf(u);
+  return -__logf(e);
 }
 
 // Reduce 16 columns held by every lane of a warp (lane l holds vocab id
 // base + l) so that lanes 2c and 2c+1 end with column c reduced over all 32
 // lanes.  Each butterfly level exchanges half of the remaining columns, so a
 // column costs about one merge per lane instead of five.
-CS_DEV Stat warp_reduce16(const float (&x)[16], int lane, int vid) {
+template <bool KEYED>
+CS_DEV Stat warp_reduce16(const float (&x)[16], const float (&key)[16], int lane, int vid) {
   Stat a[8];
   {
     const bool up = (lane & 16) != 0;
@@ -93,7 +152,13 @@ CS_DEV Stat warp_reduce16(const float (&x)[16], int lane, int vid) {
       const float send = up ? x[c] : x[c + 8];
       const float keep = up ? x[c + 8] : x[c];
       const float recv = __shfl_xor_sync(0xffffffffu, send, 16);
-      a[c] = stat_merge(stat_of(keep, vid), stat_of(recv, pv));
+      float keep_k = 0.f, recv_k = 0.f;
+      if (KEYED) {
+        const float send_k = up ? key[c] : key[c + 8];
+        keep_k = up ? key[c + 8] : key[c];
+        recv_k = __shfl_xor_sync(0xffffffffu, send_k, 16);
+      }
+      a[c] = stat_merge<KEYED>(stat_of(keep, keep_k, vid), stat_of(recv, recv_k, pv));
     }
   }
   Stat b4[4];
@@ -103,7 +168,7 @@ CS_DEV Stat warp_reduce16(const float (&x)[16], int lane, int vid) {
     for (int c = 0; c < 4; ++c) {
       const Stat send = up ? a[c] : a[c + 4];
       const Stat keep = up ? a[c + 4] : a[c];
-      b4[c] = stat_merge(keep, stat_shfl_xor(send, 8));
+      b4[c] = stat_merge<KEYED>(keep, stat_shfl_xor<KEYED>(send, 8));
     }
   }
   Stat c2[2];
@@ -113,7 +178,7 @@ CS_DEV Stat warp_reduce16(const float (&x)[16], int lane, int vid) {
     for (int c = 0; c < 2; ++c) {
       const Stat send = up ? b4[c] : b4[c + 2];
       const Stat keep = up ? b4[c + 2] : b4[c];
-      c2[c] = stat_merge(keep, stat_shfl_xor(send, 4));
+      c2[c] = stat_merge<KEYED>(keep, stat_shfl_xor<KEYED>(send, 4));
     }
   }
   Stat d1;
@@ -121,9 +186,9 @@ CS_DEV Stat warp_reduce16(const float (&x)[16], int lane, int vid) {
     const bool up = (lane & 2) != 0;
     const Stat send = up ? c2[0] : c2[1];
     const Stat keep = up ? c2[1] : c2[0];
-    d1 = stat_merge(keep, stat_shfl_xor(send, 2));
+    d1 = stat_merge<KEYED>(keep, stat_shfl_xor<KEYED>(send, 2));
   }
-  return stat_merge(d1, stat_shfl_xor(d1, 1));
+  return stat_merge<KEYED>(d1, stat_shfl_xor<KEYED>(d1, 1));
 }
 
 struct LmParams {
@@ -131,6 +196,9 @@ struct LmParams {
   float* stats;                  // [M][5]
   float4* part;                  // [gridDim.x][n_rows]: (m, sec, s, t)
   int* part_idx;                 // [gridDim.x][n_rows]
+  float* part_k;                 // [gridDim.x][n_rows], KEYED only
+  const unsigned long long* seed;  // KEYED only: Philox key (low word, high word)
+  float inv_temp;                // KEYED only: 1 / T
   int row0, n_rows, n_mma;
   int d, V, num_tiles, stages;
   uint32_t tmem_cols;
@@ -138,10 +206,12 @@ struct LmParams {
 };
 
 struct SmemLayout {
-  uint32_t a_off, b_off, bar_off, epi_off, total;
+  uint32_t a_off, b_off, bar_off, epi_off, key_off, total;
 };
 
-__host__ __device__ inline SmemLayout lm_layout(int stages, int n_mma) {
+// The KEYED tuples (per-warp keys [4][n_mma], running keys [n_mma]) go after
+// everything else, so the greedy layout is the same with or without them.
+__host__ __device__ inline SmemLayout lm_layout(int stages, int n_mma, bool keyed) {
   SmemLayout L;
   L.a_off = 0;
   L.b_off = (uint32_t)stages * A_BYTES;
@@ -149,11 +219,14 @@ __host__ __device__ inline SmemLayout lm_layout(int stages, int n_mma) {
   const uint32_t bar_bytes = (uint32_t)(2 * stages + 5) * 8 + 16;
   L.epi_off = (L.bar_off + bar_bytes + 15) / 16 * 16;
   // epilogue: per-warp tuples [4][n_mma] (float4 + int), running [n_mma] (float4 + int), draft ids
-  const uint32_t epi = 4u * n_mma * 20u + (uint32_t)n_mma * 20u + (uint32_t)n_mma * 4u + 16u;
-  L.total = L.epi_off + epi;
+  const uint32_t epi = 4u * n_mma * 20u + (uint32_t)n_mma * 20u + (uint32_t)n_mma * 4u +
+                       4u * EPI_WARPS;
+  L.key_off = L.epi_off + epi;
+  L.total = L.key_off + (keyed ? 5u * (uint32_t)n_mma * 4u : 0u);
   return L;
 }
 
+template <bool KEYED>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     lmhead_kernel(const __grid_constant__ CUtensorMap tmap_w,
                   const __grid_constant__ CUtensorMap tmap_h, const LmParams p) {
@@ -161,7 +234,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   // TMA with 128B swizzle and the UMMA descriptors need 1024-byte alignment.
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  const SmemLayout L = lm_layout(p.stages, p.n_mma);
+  const SmemLayout L = lm_layout(p.stages, p.n_mma, KEYED);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.bar_off);
   uint64_t* empty = full + p.stages;
   uint64_t* tfull = empty + p.stages;    // [2]
@@ -174,7 +247,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   float4* s_run = reinterpret_cast<float4*>(s_wti + 4 * p.n_mma);  // [n_mma]
   int* s_runi = reinterpret_cast<int*>(s_run + p.n_mma);           // [n_mma]
   int* s_draft = s_runi + p.n_mma;                                 // [n_mma]
-  volatile int* s_fail = reinterpret_cast<volatile int*>(s_draft + p.n_mma);  // [4]
+  volatile int* s_fail = reinterpret_cast<volatile int*>(s_draft + p.n_mma);  // [EPI_WARPS]
+  float* s_wk = reinterpret_cast<float*>(smem + L.key_off);         // [4][n_mma], KEYED
+  float* s_runk = s_wk + 4 * p.n_mma;                               // [n_mma], KEYED
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int kblocks = p.d / BK;
@@ -204,10 +279,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
   griddep_wait();                        // hidden rows may come from the previous kernel
+  uint32_t seed_lo = 0, seed_hi = 0;
   if (warp >= 2) {
+    if (KEYED) {
+      const unsigned long long sd = *p.seed;
+      seed_lo = (uint32_t)sd;
+      seed_hi = (uint32_t)(sd >> 32);
+    }
     for (int c = tid - 64; c < p.n_mma; c += EPI_THREADS) {
       s_run[c] = make_float4(-INFINITY, -INFINITY, 0.f, 0.f);
       s_runi[c] = 0x7fffffff;
+      if (KEYED) s_runk[c] = -INFINITY;
       s_draft[c] = (c < p.n_rows) ? p.draft_for_row[p.row0 + c] : -2;
     }
     named_bar_sync(1, EPI_THREADS);
@@ -299,18 +381,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   } else {
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;               // TMEM lane quarter this warp may access
+    const int ew = warp - 2;              // epilogue warp index
+    const int half = ew >> 2;             // which alternate 16-column chunks it takes
     const int etid = tid - 64;
     const int nchunks = (p.n_rows + 15) / 16;
     int it = 0;
     for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x, ++it) {
       const int acc = it & 1;
       const uint32_t aph = (uint32_t)(it >> 1) & 1u;
-      // The four epilogue warps take the abort decision together (named
+      // The epilogue warps take the abort decision together (named
       // barrier + shared flags) so none of them is left waiting at a barrier.
       const bool ok = __all_sync(0xffffffffu, mbar_wait(&tfull[acc], aph, WAIT_NS));
-      if (lane == 0) s_fail[q] = ok ? 0 : 1;
+      if (lane == 0) s_fail[ew] = ok ? 0 : 1;
       named_bar_sync(1, EPI_THREADS);
-      if (s_fail[0] | s_fail[1] | s_fail[2] | s_fail[3]) {
+      int any_fail = 0;
+#pragma unroll
+      for (int w = 0; w < EPI_WARPS; ++w) any_fail |= s_fail[w];
+      if (any_fail) {
         if (etid == 0) {
           set_err(p.err, ERR_TIMEOUT);
           *abort_flag = 1;
@@ -321,7 +408,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int vid = tile * BM + q * 32 + lane;
       const bool valid = vid < p.V;
       const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * p.n_mma);
-      for (int ch = 0; ch < nchunks; ++ch) {
+      for (int ch = half; ch < nchunks; ch += EPI_WARPS / 4) {
         float x[16];
         tmem_ld16(tbase + (uint32_t)(ch * 16), x);
 #pragma unroll
@@ -330,11 +417,30 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           if (valid && s_draft[col] == vid) p.stats[(size_t)(p.row0 + col) * 5 + 4] = x[c];
           if (!valid) x[c] = -INFINITY;
         }
-        const Stat r = warp_reduce16(x, lane, vid);
+        float key[16];
+        if (KEYED) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int c0 = ch * 16 + 4 * j;
+            if (c0 < p.n_rows) {             // warp-uniform
+              const uint4 u = philox4x32_10(
+                  make_uint4((uint32_t)vid, (uint32_t)((p.row0 + c0) >> 2), 0u, 0u), seed_lo, seed_hi);
+              key[4 * j + 0] = fmaf(x[4 * j + 0], p.inv_temp, gumbel_of(u.x));
+              key[4 * j + 1] = fmaf(x[4 * j + 1], p.inv_temp, gumbel_of(u.y));
+              key[4 * j + 2] = fmaf(x[4 * j + 2], p.inv_temp, gumbel_of(u.z));
+              key[4 * j + 3] = fmaf(x[4 * j + 3], p.inv_temp, gumbel_of(u.w));
+            } else {
+#pragma unroll
+              for (int c = 0; c < 4; ++c) key[4 * j + c] = -INFINITY;
+            }
+          }
+        }
+        const Stat r = warp_reduce16<KEYED>(x, key, lane, vid);
         const int col = ch * 16 + (lane >> 1);
         if ((lane & 1) == 0 && col < p.n_rows) {
           s_wt[q * p.n_mma + col] = make_float4(r.m, r.sec, r.s, r.t);
           s_wti[q * p.n_mma + col] = r.i;
+          if (KEYED) s_wk[q * p.n_mma + col] = r.k;
         }
       }
       tc_fence_before();
@@ -342,14 +448,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       named_bar_sync(1, EPI_THREADS);
       for (int col = etid; col < p.n_rows; col += EPI_THREADS) {
         const float4 rv = s_run[col];
-        Stat acc_s{rv.x, s_runi[col], rv.y, rv.z, rv.w};
+        Stat acc_s{rv.x, s_runi[col], rv.y, rv.z, rv.w, KEYED ? s_runk[col] : 0.f};
 #pragma unroll
         for (int w = 0; w < 4; ++w) {
           const float4 v = s_wt[w * p.n_mma + col];
-          acc_s = stat_merge(acc_s, Stat{v.x, s_wti[w * p.n_mma + col], v.y, v.z, v.w});
+          acc_s = stat_merge<KEYED>(acc_s, Stat{v.x, s_wti[w * p.n_mma + col], v.y, v.z, v.w,
+                                                KEYED ? s_wk[w * p.n_mma + col] : 0.f});
         }
         s_run[col] = make_float4(acc_s.m, acc_s.sec, acc_s.s, acc_s.t);
         s_runi[col] = acc_s.i;
+        if (KEYED) s_runk[col] = acc_s.k;
       }
       named_bar_sync(1, EPI_THREADS);
     }
@@ -357,6 +465,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     for (int col = etid; col < p.n_rows; col += EPI_THREADS) {
       p.part[(size_t)blockIdx.x * p.n_rows + col] = s_run[col];
       p.part_idx[(size_t)blockIdx.x * p.n_rows + col] = s_runi[col];
+      if (KEYED) p.part_k[(size_t)blockIdx.x * p.n_rows + col] = s_runk[col];
     }
   }
 
@@ -370,9 +479,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 }
 
 // Merge the per-CTA partial statistics of every row (one warp per row).
+// argmax receives the sampled id when KEYED.
+template <bool KEYED>
 __global__ void __launch_bounds__(128) lmhead_reduce_kernel(const float4* part, const int* part_idx,
-                                                            int nparts, int row0, int n_rows,
-                                                            int V, const int32_t* draft_for_row,
+                                                            const float* part_k, int nparts,
+                                                            int row0, int n_rows, int V,
+                                                            const int32_t* draft_for_row,
                                                             int32_t* argmax, float* stats, int* err) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row = blockIdx.x * 4 + warp;
@@ -382,10 +494,11 @@ __global__ void __launch_bounds__(128) lmhead_reduce_kernel(const float4* part, 
   Stat a = stat_identity();
   for (int c = lane; c < nparts; c += 32) {
     const float4 v = part[(size_t)c * n_rows + row];
-    a = stat_merge(a, Stat{v.x, part_idx[(size_t)c * n_rows + row], v.y, v.z, v.w});
+    a = stat_merge<KEYED>(a, Stat{v.x, part_idx[(size_t)c * n_rows + row], v.y, v.z, v.w,
+                                  KEYED ? part_k[(size_t)c * n_rows + row] : 0.f});
   }
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) a = stat_merge(a, stat_shfl_xor(a, off));
+  for (int off = 16; off > 0; off >>= 1) a = stat_merge<KEYED>(a, stat_shfl_xor<KEYED>(a, off));
   if (lane == 0) {
     const int m = row0 + row;
     float* st = stats + (size_t)m * 5;
@@ -423,37 +536,46 @@ LmheadPlan plan_lmhead(int M, int d, int V, int num_sms) {
   pl.passes = (M + MAX_ROWS - 1) / MAX_ROWS;
   pl.num_tiles = (V + BM - 1) / BM;
   pl.grid = pl.num_tiles < num_sms ? pl.num_tiles : num_sms;
+  // One plan serves both variants: shared memory is sized for the keyed
+  // layout, which only adds to the end of the greedy one.
   const uint32_t budget = 227u * 1024u - 1024u;
-  const uint32_t fixed = lm_layout(0, pl.n_mma).total;
+  const uint32_t fixed = lm_layout(0, pl.n_mma, true).total;
   const uint32_t per_stage = A_BYTES + (uint32_t)pl.n_mma * 128u;
   int st = (int)((budget - fixed) / per_stage);
   if (st > 12) st = 12;
+  while (st > 2 && lm_layout(st, pl.n_mma, true).total > budget) --st;
   pl.stages = st;
-  pl.smem_bytes = lm_layout(st, pl.n_mma).total + 1024;
+  pl.smem_bytes = lm_layout(st, pl.n_mma, true).total + 1024;
   const size_t per_part = (size_t)1024 * MAX_ROWS;  // upper bound on CTAs x rows
-  pl.ws_bytes = per_part * sizeof(float4) + per_part * sizeof(int);
+  pl.ws_bytes = per_part * (sizeof(float4) + sizeof(int) + sizeof(float));
   return pl;
 }
 
 cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
                           const __nv_bfloat16* w, const int32_t* draft_for_row, int32_t* argmax,
                           float* stats, void* ws, const LmheadPlan& pl, int* err,
-                          cudaStream_t stream) {
+                          cudaStream_t stream, const unsigned long long* seed, float inv_temp) {
+  const bool keyed = seed != nullptr;
   CUtensorMap map_w, map_h;
   if (!make_map(&map_w, w, (uint64_t)V, (uint64_t)d, BM)) return cudaErrorInvalidValue;
   if (!make_map(&map_h, hidden, (uint64_t)M, (uint64_t)d, (uint32_t)pl.n_mma))
     return cudaErrorInvalidValue;
-  static bool configured[64] = {false};
+  static bool configured[2][64] = {{false}};
   int dev = 0;
   cudaGetDevice(&dev);
-  if (dev < 64 && !configured[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(lmhead_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         227 * 1024);
+  if (dev < 64 && !configured[keyed][dev]) {
+    cudaError_t e = keyed ? cudaFuncSetAttribute(lmhead_kernel<true>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 227 * 1024)
+                          : cudaFuncSetAttribute(lmhead_kernel<false>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 227 * 1024);
     if (e != cudaSuccess) return e;
-    configured[dev] = true;
+    configured[keyed][dev] = true;
   }
   float4* part = static_cast<float4*>(ws);
   int* part_idx = reinterpret_cast<int*>(part + (size_t)1024 * MAX_ROWS);
+  float* part_k = reinterpret_cast<float*>(part_idx + (size_t)1024 * MAX_ROWS);
   uint32_t tmem_cols = 32;
   while (tmem_cols < (uint32_t)(2 * pl.n_mma)) tmem_cols <<= 1;
   for (int pass = 0; pass < pl.passes; ++pass) {
@@ -462,6 +584,9 @@ cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
     p.stats = stats;
     p.part = part;
     p.part_idx = part_idx;
+    p.part_k = part_k;
+    p.seed = seed;
+    p.inv_temp = inv_temp;
     p.row0 = pass * MAX_ROWS;
     p.n_rows = (M - p.row0) < MAX_ROWS ? (M - p.row0) : MAX_ROWS;
     p.n_mma = pl.n_mma;
@@ -471,12 +596,23 @@ cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
     p.stages = pl.stages;
     p.tmem_cols = tmem_cols;
     p.err = err;
-    cudaError_t e = launch_pdl(lmhead_kernel, dim3(pl.grid), dim3(NUM_THREADS), pl.smem_bytes,
-                               stream, map_w, map_h, p);
-    if (e != cudaSuccess) return e;
-    e = launch_pdl(lmhead_reduce_kernel, dim3((p.n_rows + 3) / 4), dim3(128), 0, stream,
-                   (const float4*)part, (const int*)part_idx, pl.grid, p.row0, p.n_rows, V,
-                   draft_for_row, argmax, stats, err);
+    const dim3 rgrid((p.n_rows + 3) / 4);
+    cudaError_t e;
+    if (keyed) {
+      e = launch_pdl(lmhead_kernel<true>, dim3(pl.grid), dim3(NUM_THREADS), pl.smem_bytes, stream,
+                     map_w, map_h, p);
+      if (e != cudaSuccess) return e;
+      e = launch_pdl(lmhead_reduce_kernel<true>, rgrid, dim3(128), 0, stream, (const float4*)part,
+                     (const int*)part_idx, (const float*)part_k, pl.grid, p.row0, p.n_rows, V,
+                     draft_for_row, argmax, stats, err);
+    } else {
+      e = launch_pdl(lmhead_kernel<false>, dim3(pl.grid), dim3(NUM_THREADS), pl.smem_bytes, stream,
+                     map_w, map_h, p);
+      if (e != cudaSuccess) return e;
+      e = launch_pdl(lmhead_reduce_kernel<false>, rgrid, dim3(128), 0, stream, (const float4*)part,
+                     (const int*)part_idx, (const float*)nullptr, pl.grid, p.row0, p.n_rows, V,
+                     draft_for_row, argmax, stats, err);
+    }
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
@@ -550,7 +686,7 @@ extern "C" COSPEC_API int cospec_lmhead_argmax_features_noalloc(
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 64 && !configured[dev]) {
-    if (cudaFuncSetAttribute(lmhead_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(lmhead_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              227 * 1024) != cudaSuccess)
       return COSPEC_ERR_CUDA;
     configured[dev] = true;
@@ -574,12 +710,12 @@ extern "C" COSPEC_API int cospec_lmhead_argmax_features_noalloc(
     p.stages = pl.stages;
     p.tmem_cols = tmem_cols;
     p.err = err;
-    if (launch_pdl(lmhead_kernel, dim3(pl.grid), dim3(NUM_THREADS), pl.smem_bytes, st, map_w,
-                   map_h, p) != cudaSuccess)
+    if (launch_pdl(lmhead_kernel<false>, dim3(pl.grid), dim3(NUM_THREADS), pl.smem_bytes, st,
+                   map_w, map_h, p) != cudaSuccess)
       return COSPEC_ERR_CUDA;
-    if (launch_pdl(lmhead_reduce_kernel, dim3((p.n_rows + 3) / 4), dim3(128), 0, st,
-                   (const float4*)part, (const int*)part_idx, pl.grid, p.row0, p.n_rows, V,
-                   draft_for_row, argmax, stats, err) != cudaSuccess)
+    if (launch_pdl(lmhead_reduce_kernel<false>, dim3((p.n_rows + 3) / 4), dim3(128), 0, st,
+                   (const float4*)part, (const int*)part_idx, (const float*)nullptr, pl.grid,
+                   p.row0, p.n_rows, V, draft_for_row, argmax, stats, err) != cudaSuccess)
       return COSPEC_ERR_CUDA;
   }
   return COSPEC_OK;

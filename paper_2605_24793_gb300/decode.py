@@ -1,6 +1,8 @@
 """Multi-round CoSpec decoding on the device (App. F, Inference Procedure:
 draft, verify, arbitrate, stop at the first rejected mismatch, commit,
 repeat) and the mean accepted length tau = (1/R) sum_r s^(r) (Sec. 3.1, Eq. 5).
+With a temperature, target candidates are drawn by sampling (stochastic
+decoding, Sec. 3.1) with a fresh seed per round from a device table.
 
 The rounds reuse one CUDA graph: every replay copies that round's draft ids
 from a device table (selected by a device-side round counter), runs the
@@ -11,6 +13,7 @@ block (Q, block K/V, hidden rows) are the workload's synthetic tensors.
 
   python -m paper_2605_24793_gb300.decode --config qwen3_8b_b1 --rounds 64
   python -m paper_2605_24793_gb300.decode --sweep        # K and lambda sweep
+  python -m paper_2605_24793_gb300.decode --temperature 1
 """
 from __future__ import annotations
 
@@ -39,7 +42,7 @@ def target_ranked_ids(cfg: W.RoundConfig, hidden: torch.Tensor, w: torch.Tensor,
 class MultiRoundDecoder:
     def __init__(self, cfg: W.RoundConfig, rounds: int, lam: Optional[float] = None,
                  mode: int = C.POLICY_MLP, device="cuda", inputs: Optional[Dict] = None,
-                 drafts: Optional[np.ndarray] = None):
+                 drafts: Optional[np.ndarray] = None, temperature: Optional[float] = None):
         self.cfg, self.rounds = cfg, rounds
         self.lam = cfg.lam if lam is None else lam
         self.inp = inputs if inputs is not None else W.make_round_inputs(
@@ -50,12 +53,16 @@ class MultiRoundDecoder:
         self.drafts_np = drafts
         dev = self.inp["q"].device
         max_ctx = int(self.inp["ctx_len_np"].max()) + rounds * cfg.rows
-        self.rnd = VerifyRound(self.inp, drafts[0], self.lam, mode, max_ctx=max_ctx)
+        self.temperature = temperature
+        self.seeds_np = np.array([W.sample_seed(cfg, r) for r in range(rounds)], dtype=np.int64)
+        self.rnd = VerifyRound(self.inp, drafts[0], self.lam, mode, max_ctx=max_ctx,
+                               temperature=temperature, seed=int(self.seeds_np[0]))
         B, K, R = cfg.batch, cfg.k, cfg.rows
         dfr = np.full((rounds, B, R), -1, dtype=np.int32)
         dfr[:, :, :K] = drafts
         self.drafts = torch.from_numpy(np.ascontiguousarray(drafts, dtype=np.int32)).to(dev)
         self.dfr = torch.from_numpy(dfr.reshape(rounds, B * R)).to(dev)
+        self.seeds = torch.from_numpy(self.seeds_np).to(dev)
         self.idx = torch.zeros(1, dtype=torch.int64, device=dev)
         self.s_hist = torch.zeros((rounds, B), dtype=torch.int32, device=dev)
         self.emitted_hist = torch.full((rounds, B, R), -1, dtype=torch.int32, device=dev)
@@ -65,6 +72,8 @@ class MultiRoundDecoder:
         B, K = self.cfg.batch, self.cfg.k
         torch.index_select(self.drafts, 0, self.idx, out=self.rnd.draft.view(1, B, K))
         torch.index_select(self.dfr, 0, self.idx, out=self.rnd.draft_for_row.view(1, -1))
+        if self.temperature is not None:
+            torch.index_select(self.seeds, 0, self.idx, out=self.rnd.seed)
         self.rnd.run(restore=False)
         self.s_hist.index_copy_(0, self.idx, self.rnd.accept_len.view(1, B))
         self.emitted_hist.index_copy_(0, self.idx, self.rnd.emitted.view(1, B, -1))
@@ -118,6 +127,8 @@ def main():
     ap.add_argument("--rounds", type=int, default=64)
     ap.add_argument("--k", type=int, default=None)
     ap.add_argument("--lam", type=float, default=None)
+    ap.add_argument("--temperature", type=float, default=None,
+                    help="sample target candidates at this temperature (default: greedy)")
     ap.add_argument("--sweep", action="store_true",
                     help="K in {15, 20, 25} at lambda 0.6, then lambda in {0.4, 0.6, 0.8} at K 25")
     args = ap.parse_args()
@@ -131,9 +142,10 @@ def main():
         points = [(args.k if args.k is not None else base.k, args.lam if args.lam is not None else base.lam)]
     for k, lam in points:
         cfg = base.replace(k=k)
-        dec = MultiRoundDecoder(cfg, args.rounds, lam)
+        dec = MultiRoundDecoder(cfg, args.rounds, lam, temperature=args.temperature)
         res = dec.run()
-        res.update({"workload": cfg.name, "k": k, "lambda": lam, "batch": cfg.batch})
+        res.update({"workload": cfg.name, "k": k, "lambda": lam, "batch": cfg.batch,
+                    "temperature": args.temperature})
         print(json.dumps(res), flush=True)
         del dec
         torch.cuda.empty_cache()

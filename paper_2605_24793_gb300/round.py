@@ -19,7 +19,12 @@ from . import cospec as C
 
 class VerifyRound:
     def __init__(self, inputs: Dict[str, object], draft: np.ndarray, lam: float = 0.6,
-                 mode: int = C.POLICY_MLP, keep_attn: bool = False, max_ctx: Optional[int] = None):
+                 mode: int = C.POLICY_MLP, keep_attn: bool = False, max_ctx: Optional[int] = None,
+                 temperature: Optional[float] = None, seed: int = 0):
+        """``temperature`` None: greedy target candidates (argmax).  Otherwise
+        stochastic decoding (Sec. 3.1): candidates are Gumbel-max samples at
+        that temperature, keyed by the device scalar ``self.seed``, which a
+        caller may rewrite between replays of a captured round."""
         cfg = inputs["cfg"]
         self.cfg = cfg
         self.inp = inputs
@@ -50,6 +55,8 @@ class VerifyRound:
         self.accept = torch.empty((B, K), dtype=torch.uint8, device=dev)
         self.accept_len = torch.empty(B, dtype=torch.int32, device=dev)
         self.emitted = torch.empty((B, R), dtype=torch.int32, device=dev)
+        self.temperature = None if temperature is None else float(temperature)
+        self.seed = torch.tensor([int(seed)], dtype=torch.int64, device=dev)
         self.graph: Optional[torch.cuda.CUDAGraph] = None
         self.launches_per_round = self._count_launches()
 
@@ -75,6 +82,10 @@ class VerifyRound:
                              kv_stable=l > 0)
 
     def lmhead(self):
+        if self.temperature is not None:
+            return C.lmhead_sample_features(self.hidden, self.w, self.draft_for_row,
+                                            self.temperature, self.seed, self.argmax, self.stats,
+                                            self.ws_lm)
         return C.lmhead_argmax_features(self.hidden, self.w, self.draft_for_row, self.argmax,
                                         self.stats, self.ws_lm)
 

@@ -34,7 +34,7 @@ import torch
 
 # tensor ids used in the seed formula config.index * 1000 + id
 _TID = dict(ctx=1, pages=2, q=3, k_blk=4, v_blk=5, k_pages=6, v_pages=7,
-            hidden=8, w=9, mlp=10, drafts=11)
+            hidden=8, w=9, mlp=10, drafts=11, sample=12)
 
 NUM_FEATURES = 8
 
@@ -268,6 +268,12 @@ def synth_drafts(cfg: RoundConfig, ranked_ids: np.ndarray, round_index: int = 0)
                 other = int(rng.integers(0, cfg.vocab - 1))
                 draft[b, i] = other + (other >= top1)
     return draft
+
+
+def sample_seed(cfg: RoundConfig, round_index: int = 0) -> int:
+    """64-bit key of round ``round_index``'s sampling noise (stochastic
+    decoding); both words vary with the round."""
+    return (seed_of(cfg, "sample") + round_index) * 0x9E3779B97F4A7C15 % (1 << 63)
 
 
 def draft_for_rows(draft: np.ndarray) -> np.ndarray:

@@ -32,12 +32,15 @@ def assert_close(got, ref, what: str, abs_tol: float = TOL_ABS, rel_tol: float =
     return float(err.max()) if err.size else 0.0
 
 
-def tie_affected(ref_stats, ref_draft, ref_argmax, ref_p, s_ref, s_gpu, lam):
+def tie_affected(ref_stats, ref_draft, ref_argmax, ref_p, s_ref, s_gpu, lam, margin=None):
     """Per-sequence tie flags.  ref_stats [B,R,5], ref_draft [B,K],
-    ref_argmax [B,R], ref_p [B,K], s_* [B]."""
+    ref_argmax [B,R], ref_p [B,K], s_* [B].  ``margin`` [B,R] overrides the
+    top-1/top-2 logit gap (for sampled candidates: the gap of the perturbed
+    keys)."""
     B, R = ref_argmax.shape
     K = R - 1
-    margin = ref_stats[:, :, 0] - ref_stats[:, :, 1]
+    if margin is None:
+        margin = ref_stats[:, :, 0] - ref_stats[:, :, 1]
     flags = np.zeros(B, dtype=bool)
     for b in range(B):
         reach = min(K, int(max(s_ref[b], s_gpu[b])))

@@ -104,3 +104,18 @@ def test_commit_host_validation(lib):
     # layer stride smaller than one pool
     assert f(2, 5, 36, ctypes.byref(d), *args, 1024, fake, fake, fake, fake, None) == -1
     assert f(2, 5, 36, ctypes.byref(d), *([None] * 7), 10 ** 9, fake, fake, fake, fake, None) == -1
+
+
+def test_sample_host_validation(lib):
+    f = lib.cospec_lmhead_sample_features
+    fake = ctypes.c_void_p(1 << 20)
+    args = lambda T, seed: (4, 4096, 1000, fake, fake, fake, T, seed, fake, fake, fake, 1 << 30, None)
+    assert f(*args(0.0, fake)) == -1                                  # temperature must be > 0
+    assert f(*args(-1.0, fake)) == -1
+    assert f(*args(float("nan"), fake)) == -1
+    assert f(*args(float("inf"), fake)) == -1
+    assert f(*args(1e-45, fake)) == -1                                # 1 / T overflows
+    assert f(*args(1.0, None)) == -1                                  # seed pointer missing
+    assert f(*args(1.0, ctypes.c_void_p((1 << 20) + 4))) == -1        # seed not 8-byte aligned
+    assert f(0, 4096, 1000, *([None] * 3), 1.0, None, None, None, None, 0, None) == 0
+    assert f(4, 4000, 1000, fake, fake, fake, 1.0, fake, fake, fake, fake, 1 << 30, None) == -2

@@ -344,3 +344,148 @@ def test_device_checks_set_error_bits_without_faulting():
                              C.new_lmhead_workspace(M, d, V))
     assert C.get_device_error() == C.DEVERR_TOKEN
     assert C.get_device_error() == 0                       # reading clears the word
+
+
+# ---------------------------------------------------------------------------
+# Stochastic decoding: temperature sampling in the LM-head epilogue (Sec. 3.1)
+# ---------------------------------------------------------------------------
+
+def _key_margin(keys: np.ndarray) -> np.ndarray:
+    top2 = np.sort(keys, axis=1)[:, -2:]
+    return top2[:, 1] - top2[:, 0]
+
+
+SAMPLE_CASES = [
+    # M, d, V, weight std, temperature, seed
+    (1, 64, 128, 0.1, 1.0, 0),
+    (6, 4096, 151936, 0.02, 1.0, 0x0123456789ABCDEF),   # Qwen3-8B LM head, batch 1, K = 5
+    (17, 256, 1000, 0.1, 0.5, 7),                      # ragged vocabulary tile, rows not 4-aligned
+    (300, 128, 2048, 0.1, 1.0, 2 ** 40 + 3),           # two 256-row passes
+    (64, 512, 4096, 0.3, 2.0, 99),
+]
+
+
+@pytest.mark.parametrize("case", SAMPLE_CASES, ids=lambda c: f"M{c[0]}V{c[2]}T{c[4]}")
+def test_lmhead_sampling_matches_oracle(case):
+    M, d, V, wstd, T, seed = case
+    rng = np.random.default_rng(M * 13 + V)
+    hidden = bf16(rng.standard_normal((M, d)))
+    w = bf16(rng.standard_normal((V, d)) * wstd)
+    dfr = rng.integers(-1, V, M).astype(np.int32)
+    smp = torch.empty(M, dtype=torch.int32, device="cuda")
+    st = torch.empty((M, 5), dtype=torch.float32, device="cuda")
+    seed_t = torch.tensor([seed], dtype=torch.int64, device="cuda")
+    C.lmhead_sample_features(hidden, w, torch.from_numpy(dfr).cuda(), T, seed_t, smp, st,
+                             C.new_lmhead_workspace(M, d, V))
+    x = O.lmhead_logits(host(hidden), host(w))
+    ref_s, ref_st = O.row_stats_sampled(x, dfr, seed, T)
+    assert_close(st.cpu().numpy(), ref_st, "sampled lm-head stats")
+    clear = _key_margin(O.gumbel_keys(x, seed, T)) >= 1e-3
+    got = smp.cpu().numpy()
+    assert np.array_equal(got[clear], ref_s[clear])
+    assert np.all((got >= 0) & (got < V))
+    # with this much noise the sample is often not the argmax
+    if M >= 17:
+        assert np.mean(got != np.argmax(x, axis=1)) > 0.2
+    print(f"sampled lm-head {case}: tie rows {(~clear).sum()}")
+
+
+def test_lmhead_sampling_reads_the_seed_when_the_graph_runs():
+    M, d, V = 12, 256, 3000
+    rng = np.random.default_rng(5)
+    hidden = bf16(rng.standard_normal((M, d)))
+    w = bf16(rng.standard_normal((V, d)) * 0.05)
+    dfr = torch.full((M,), -1, dtype=torch.int32, device="cuda")
+    smp = torch.empty(M, dtype=torch.int32, device="cuda")
+    st = torch.empty((M, 5), dtype=torch.float32, device="cuda")
+    seed_t = torch.tensor([1], dtype=torch.int64, device="cuda")
+    ws = C.new_lmhead_workspace(M, d, V)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        C.lmhead_sample_features(hidden, w, dfr, 1.0, seed_t, smp, st, ws)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        C.lmhead_sample_features(hidden, w, dfr, 1.0, seed_t, smp, st, ws)
+    x = O.lmhead_logits(host(hidden), host(w))
+    seen = []
+    for seed in (3, 2 ** 33 + 5, 12345):
+        seed_t.fill_(seed)
+        g.replay()
+        torch.cuda.synchronize()
+        got = smp.cpu().numpy()
+        ref, _ = O.row_stats_sampled(x, np.full(M, -1), seed, 1.0)
+        clear = _key_margin(O.gumbel_keys(x, seed, 1.0)) >= 1e-3
+        assert np.array_equal(got[clear], ref[clear])
+        seen.append(got)
+    assert not np.array_equal(seen[0], seen[1]) and not np.array_equal(seen[1], seen[2])
+
+
+def test_lmhead_sampling_at_tiny_temperature_is_the_argmax():
+    M, d, V = 40, 512, 5000
+    rng = np.random.default_rng(8)
+    hidden = bf16(rng.standard_normal((M, d)))
+    w = bf16(rng.standard_normal((V, d)) * 0.05)
+    dfr = torch.full((M,), -1, dtype=torch.int32, device="cuda")
+    ws = C.new_lmhead_workspace(M, d, V)
+    am = torch.empty(M, dtype=torch.int32, device="cuda")
+    smp = torch.empty(M, dtype=torch.int32, device="cuda")
+    st0 = torch.empty((M, 5), dtype=torch.float32, device="cuda")
+    st1 = torch.empty((M, 5), dtype=torch.float32, device="cuda")
+    C.lmhead_argmax_features(hidden, w, dfr, am, st0, ws)
+    C.lmhead_sample_features(hidden, w, dfr, 1e-5, torch.tensor([77], dtype=torch.int64,
+                             device="cuda"), smp, st1, ws)
+    x = O.lmhead_logits(host(hidden), host(w))
+    top2 = np.sort(x, axis=1)[:, -2:]
+    clear = (top2[:, 1] - top2[:, 0]) >= 1e-3
+    assert np.array_equal(smp.cpu().numpy()[clear], am.cpu().numpy()[clear])
+    # the statistics do not depend on the sampling (up to the summation order on exact ties)
+    torch.testing.assert_close(st0, st1, rtol=1e-6, atol=1e-6, equal_nan=True)
+
+
+@pytest.mark.parametrize("T", [1.0, 0.6])
+def test_tiny_sampled_round_matches_oracle(T):
+    cfg = W.CONFIGS["tiny"].replace(batch=3, k=6, mismatch_rate=0.5, ctx_lo=30, ctx_hi=200,
+                                    shuffled_pages=True)
+    inp = W.make_round_inputs(cfg, device="cuda")
+    hostd = {kk: (v.cpu() if torch.is_tensor(v) else v) for kk, v in inp.items()}
+    x = O.lmhead_logits(hostd["hidden"], hostd["w"])
+    ranked = O.topk_ids(x, 8).reshape(cfg.batch, cfg.rows, 8)
+    draft = W.synth_drafts(cfg, ranked)
+    seed = W.sample_seed(cfg, 0)
+    rnd = VerifyRound(inp, draft, cfg.lam, C.POLICY_MLP, temperature=T, seed=seed)
+    rnd.run()
+    torch.cuda.synchronize()
+    ref = O.cospec_round(hostd, draft, cfg.lam, with_attention=False, with_commit=False,
+                         sample_seed=seed, temperature=T)
+    s_gpu = rnd.accept_len.cpu().numpy()
+    tie = tie_affected(ref["stats"], draft, ref["argmax"], ref["p"], ref["s"], s_gpu, cfg.lam,
+                       margin=ref["key_margin"])
+    ok = ~tie
+    assert np.array_equal(s_gpu[ok], ref["s"][ok])
+    assert np.array_equal(rnd.emitted.cpu().numpy().reshape(cfg.batch, -1)[ok], ref["emitted"][ok])
+    clear = ref["key_margin"] >= 1e-3
+    assert np.array_equal(rnd.argmax.cpu().numpy().reshape(cfg.batch, -1)[clear],
+                          ref["argmax"][clear])
+    print(f"sampled round T={T}: s {s_gpu.tolist()} ties {int(tie.sum())}")
+
+
+def test_lmhead_sampling_noise_only_at_huge_temperature():
+    """At T = 1e6 the keys are the Gumbel noise alone (|x / T| < 1e-5), so each
+    row's sample is the position of the largest of V noise values: the
+    generator, the counter layout and the upper tail of g are checked against
+    the oracle's float64 noise directly."""
+    M, d, V, T, seed = 64, 256, 20000, 1e6, 0xDEADBEEF12345
+    rng = np.random.default_rng(21)
+    hidden = bf16(rng.standard_normal((M, d)))
+    w = bf16(rng.standard_normal((V, d)) * 0.01)
+    smp = torch.empty(M, dtype=torch.int32, device="cuda")
+    st = torch.empty((M, 5), dtype=torch.float32, device="cuda")
+    C.lmhead_sample_features(hidden, w, torch.full((M,), -1, dtype=torch.int32, device="cuda"), T,
+                             torch.tensor([seed], dtype=torch.int64, device="cuda"), smp, st,
+                             C.new_lmhead_workspace(M, d, V))
+    x = O.lmhead_logits(host(hidden), host(w))
+    keys = O.gumbel_keys(x, seed, T)
+    clear = _key_margin(keys) >= 1e-3
+    assert clear.sum() >= M - 2
+    assert np.array_equal(smp.cpu().numpy()[clear], np.argmax(keys, axis=1)[clear])
