@@ -53,20 +53,21 @@ struct Layout {
   static constexpr int PD = D + 8;                 // padded fp32 row of a partial (no bank conflicts)
   static constexpr int ROWP = PD * 4;              // bytes of a partial row: O[D], (m, l), pad
   static constexpr int RED = (WK > 1) ? MT * WK * 16 * ROWP : 0;
-  // Partials pushed by the cluster's CTAs land in RECV [S][rows per owner]
-  // (at most NRP rows in all); it overlaps RED and the ring, which are idle
-  // by then.  PART, this CTA's own partial [NRP rows], lies beyond both.
-  static constexpr int RECV = 0;
-  static constexpr bool CAN_SPLIT =
-      (RED > NRP * ROWP ? RED : NRP * ROWP) + NRP * ROWP <= NSTAGE * STAGE;   // else one CTA
-  static constexpr int PART = CAN_SPLIT ? (RED > NRP * ROWP ? RED : NRP * ROWP) : RED;
+  // After the last tile the ring holds, in order: RED (per-warp partials
+  // when keys are split over warps), PART (this CTA's partial, NRP rows) and
+  // RECV [S][rows per owner] (S * ceil(NR / S) <= NRP + 15 rows), where the
+  // cluster's CTAs push their partials.  RECV overlaps neither RED nor PART,
+  // so peers may push while this CTA still reduces its own partial.
+  static constexpr int PART = RED;
   static constexpr int PART_END = PART + NRP * ROWP;
+  static constexpr int RECV = PART_END;
+  static constexpr int RECV_END = RECV + (NRP + 15) * ROWP;
+  static_assert(RECV_END <= NSTAGE * STAGE, "partials must fit in the stage ring");
   static constexpr int BAR = NSTAGE * STAGE;       // full[NSTAGE], empty[NSTAGE], block
   static constexpr int BLK = BAR + (2 * NSTAGE + 2) * 8 + 1024;   // 1024-aligned block K/V
   // the block region holds 2*H halves of KBR rows (KBR = 16 or 32, runtime)
   static constexpr int blk_half(int kbr) { return kbr * ROWB; }
   static constexpr int total(int kbr) { return BLK / 1024 * 1024 + 2 * H * kbr * ROWB; }
-  static_assert(PART_END <= NSTAGE * STAGE, "partials must fit in the stage ring");
 };
 
 // Shared-memory byte offset of 16-byte chunk `ch` (of D/8) of key row `key`
@@ -401,6 +402,13 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
     l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
   }
   __syncthreads();
+  // The ring is idle from here on.  Tell the cluster (its CTAs may push into
+  // RECV once every CTA has arrived) and build this CTA's partial meanwhile.
+  const int rpo = (NR + S - 1) / S;      // rows finished by each owner
+  if (S > 1) {
+    if (tid == 0) mbar_arrive_expect_tx(recv_bar, (uint32_t)(S * rpo * LY::ROWP));
+    cluster_arrive();
+  }
 
   // CTA partial: rows of every warp, key groups merged (stage ring reused).
   // A partial row holds O[0..D) then (m, l) at D, D+1 (fp32, padded to PD).
@@ -477,11 +485,9 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
   // Each CTA sends its partial rows to their owners with one bulk shared-
   // to-shared copy per owner (thread-level remote accesses are slow); the
   // owner merges the S received copies from its own shared memory.
-  const int rpo = (NR + S - 1) / S;
   const float* src = part;
   if (S > 1) {
-    if (tid == 0) mbar_arrive_expect_tx(recv_bar, (uint32_t)(S * rpo * LY::ROWP));
-    cluster_sync();                      // peers' rings / reduction buffers are idle now
+    cluster_wait();                      // every CTA's RECV is free and its barrier armed
     float* recv = reinterpret_cast<float*>(smem + LY::RECV);   // [S][rpo][PD] at each owner
     if (tid == 0) {
       const uint32_t recv_u = smem_u32(recv), bar_u = smem_u32(recv_bar);
@@ -492,6 +498,10 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
     }
     if (!mbar_wait(recv_bar, 0)) set_err(p.err, ERR_TIMEOUT);
     src = recv;
+    // Everything addressed to this CTA has landed.  Once every CTA has said
+    // so, no copy reads or writes this CTA's shared memory any more: arrive
+    // now, wait at the very end, and merge in between.
+    cluster_arrive();
   }
   const int row0 = rank * rpo;
   for (int e = tid; e < rpo * (D / 4); e += NTT) {
@@ -522,7 +532,7 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
     pk.y = pack_bf16(acc.z * inv, acc.w * inv);
     *reinterpret_cast<uint2*>(dst) = pk;
   }
-  if (S > 1) cluster_sync();             // every copy out of this CTA has landed
+  if (S > 1) cluster_wait();             // every copy out of this CTA has landed
 }
 
 
