@@ -99,7 +99,10 @@ COSPEC_API int cospec_num_sms(void);
  *    max_ctx  an upper bound of ctx_len[*] (host-side; sizes the KV split)
  *    No workspace: the KV range of a (sequence, KV head) is split over the
  *    CTAs of one thread-block cluster, whose partial results merge in
- *    distributed shared memory.
+ *    distributed shared memory.  Two kernels implement the call: one on
+ *    mma.sync tensor-core tiles, and one on tcgen05 (TMEM accumulators),
+ *    used when a KV head's group has more than 32 query rows and the batch
+ *    gives every SM a (sequence, KV head, row group) of its own.
  *    Supported: head_dim in {64, 128}; page_size == 16; rows <= 32;
  *    num_q_heads % num_kv_heads == 0; (num_q_heads / num_kv_heads) * rows <= 512.
  * ------------------------------------------------------------------------ */
@@ -121,6 +124,13 @@ typedef struct {
  * when that kernel writes none of them (e.g. between the layers of one
  * round, where only q / k_blk / v_blk come from the previous layer). */
 #define COSPEC_ATTN_KV_STABLE 1
+
+/* Launch plan cospec_verify_attn would use for these dimensions on the
+ * current device: *kernel = 0 (mma.sync) or 1 (tcgen05), *splits = CTAs per
+ * (sequence, KV head, row group).  Host only; returns COSPEC_OK or the error
+ * cospec_verify_attn would return for the dimensions. */
+COSPEC_API int cospec_verify_attn_plan(const cospec_attn_dims* dims, int max_ctx, int* kernel,
+                                       int* splits);
 
 COSPEC_API int cospec_verify_attn(const cospec_attn_dims* dims, int max_ctx,
                                   const uint16_t* q, const uint16_t* k_blk, const uint16_t* v_blk,

@@ -22,7 +22,7 @@ DEVERR_PAGE, DEVERR_CTX, DEVERR_TOKEN, DEVERR_TIMEOUT = 1, 2, 4, 8
 EXPORTED = ("cospec_status_string", "cospec_get_device_error", "cospec_num_sms",
             "cospec_verify_attn", "cospec_lmhead_workspace", "cospec_lmhead_argmax_features",
             "cospec_arbitrate", "cospec_accept_commit", "cospec_lmhead_argmax_features_noalloc",
-            "cospec_lmhead_sample_features")
+            "cospec_lmhead_sample_features", "cospec_verify_attn_plan")
 
 
 class AttnDims(ctypes.Structure):
@@ -59,6 +59,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "cospec_get_device_error": (_i, [ctypes.POINTER(_i), _vp]),
         "cospec_num_sms": (_i, []),
         "cospec_verify_attn": (_i, [_PDIMS, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
+        "cospec_verify_attn_plan": (_i, [_PDIMS, _i, ctypes.POINTER(_i), ctypes.POINTER(_i)]),
         "cospec_lmhead_workspace": (_sz, [_i, _i, _i]),
         "cospec_lmhead_argmax_features": (_i, [_i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
         "cospec_lmhead_argmax_features_noalloc": (_i, [_i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp]),
@@ -115,6 +116,18 @@ def attn_dims(q: torch.Tensor, k_pages: torch.Tensor, page_table: torch.Tensor,
 
 def num_sms() -> int:
     return load_library().cospec_num_sms()
+
+
+ATTN_MMA_SYNC, ATTN_TCGEN05 = 0, 1
+
+
+def verify_attn_plan(q, k_pages, page_table, max_ctx: int):
+    """(kernel, splits) cospec_verify_attn would use for these tensors."""
+    dims = attn_dims(q, k_pages, page_table)
+    kernel, splits = ctypes.c_int(), ctypes.c_int()
+    _check(load_library().cospec_verify_attn_plan(ctypes.byref(dims), int(max_ctx),
+                                                  ctypes.byref(kernel), ctypes.byref(splits)))
+    return kernel.value, splits.value
 
 
 def verify_attn(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len, out, max_ctx,

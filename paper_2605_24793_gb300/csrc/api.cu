@@ -140,21 +140,40 @@ static int check_attn_dims(const cospec_attn_dims* d) {
 
 // Largest schedulable cluster not above `S` for this variant (cached per device).
 static int schedulable_cluster(int D, const AttnPlan& pl, int Hkv, int B) {
-  static int cache[64][2][4][5];   // [dev][D==128][mt index][log2 S] : 0 unknown, 1 ok, -1 no
+  static int cache[64][2][6][5];   // [dev][D==128][variant][log2 S] : 0 unknown, 1 ok, -1 no
   int dev = 0;
   cudaGetDevice(&dev);
   const int di = D == 128 ? 1 : 0;
-  const int mi = pl.mt == 1 ? 0 : pl.mt == 2 ? 1 : pl.mt == 4 ? 2 : 3;
+  const int mi = pl.kind == 1 ? (pl.nt == 32 ? 4 : 5)
+                              : (pl.mt == 1 ? 0 : pl.mt == 2 ? 1 : pl.mt == 4 ? 2 : 3);
   int S = pl.cluster;
   while (S > 1) {
     int ls = 0;
     while ((1 << ls) < S) ++ls;
     int& c = cache[dev < 64 ? dev : 63][di][mi][ls];
-    if (c == 0) c = attn_max_active_clusters(D, pl.mt, pl.wk, S, Hkv, B) > 0 ? 1 : -1;
+    if (c == 0)
+      c = (pl.kind == 1 ? attn_tc_max_active_clusters(D, pl.nt, S, Hkv, B, pl.rg)
+                        : attn_max_active_clusters(D, pl.mt, pl.wk, S, Hkv, B)) > 0 ? 1 : -1;
     if (c > 0) break;
     S >>= 1;
   }
   return S;
+}
+
+COSPEC_API int cospec_verify_attn_plan(const cospec_attn_dims* d, int max_ctx, int* kernel,
+                                       int* splits) {
+  const int st = check_attn_dims(d);
+  if (st != COSPEC_OK) return st;
+  CS_CHECK_ARG(kernel && splits);
+  CS_CHECK_ARG(max_ctx >= 0 && max_ctx <= d->max_pages_per_seq * d->page_size);
+  const int sms = device_num_sms();
+  if (sms <= 0) return COSPEC_ERR_CUDA;
+  AttnPlan pl = plan_verify_attn(d->batch, d->rows, d->num_q_heads, d->num_kv_heads,
+                                 d->head_dim, max_ctx, sms);
+  pl.cluster = schedulable_cluster(d->head_dim, pl, d->num_kv_heads, d->batch);
+  *kernel = pl.kind;
+  *splits = pl.cluster;
+  return COSPEC_OK;
 }
 
 COSPEC_API int cospec_verify_attn(const cospec_attn_dims* d, int max_ctx, const uint16_t* q,

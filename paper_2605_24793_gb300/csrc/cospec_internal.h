@@ -53,8 +53,11 @@ struct AttnArgs {
   int kv_stable;   // cache-side reads may start before the previous kernel finishes
 };
 struct AttnPlan {
-  int mt, wk, nrp;
-  int cluster;            // CTAs per (sequence, KV head): the KV split
+  int kind;               // 0: mma.sync kernel, 1: tcgen05 kernel
+  int mt, wk, nrp;        // mma.sync: row tiles, key groups, padded rows
+  int nt, jb, jbq, rg;    // tcgen05: row capacity (32 / 64), block rows per row group,
+                          // block rows of the query box, row groups
+  int cluster;            // CTAs per (sequence, KV head, row group): the KV split
   int tiles_per_split, max_splits;
   size_t total_bytes;     // workspace (none)
 };
@@ -62,6 +65,10 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
 int attn_max_active_clusters(int D, int mt, int wk, int S, int Hkv, int B);
 cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& plan, int* err,
                                cudaStream_t stream);
+bool tc_attn_supported(int D, int G);
+int attn_tc_max_active_clusters(int D, int nt, int S, int Hkv, int B, int RG);
+cudaError_t launch_verify_attn_tc(const AttnArgs& a, const AttnPlan& plan, int* err,
+                                  cudaStream_t stream);
 
 // ---------------------------------------------------------------- LM head
 struct LmheadPlan {

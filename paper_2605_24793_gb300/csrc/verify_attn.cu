@@ -624,10 +624,39 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
   const long long want = want_wave > want_len ? want_wave : want_len;
   int S = 1;
   while (S < 16 && S < want && (S * 2) * 4 <= tiles) S *= 2;
+  pl.kind = 0;
   pl.cluster = S;
   pl.tiles_per_split = (tiles + S - 1) / S;
   pl.max_splits = S;
   pl.total_bytes = 0;
+  const int G = Hq / Hkv;
+  const int jb = G <= 64 ? 64 / G : 1;
+  const int jbq = R < jb ? R : jb;
+  // More than 32 query rows per group and at least one (sequence, head, row
+  // group) per SM: the mma.sync kernel is bound by its legacy tensor-core
+  // rate there, and the tcgen05 kernel (one CTA per SM, deep ring) takes
+  // over.  Small batches stay latency-bound and keep the mma.sync kernel.
+  const long long units_g = (long long)B * Hkv * ((R + jb - 1) / jb);
+  if (tc_attn_supported(D, G) && G * jbq > 32 && units_g >= num_sms) {
+    // tcgen05 kernel: row groups of whole block rows, at most 64 query rows
+    pl.kind = 1;
+    pl.jb = jb;
+    pl.jbq = jbq;
+    pl.rg = (R + pl.jb - 1) / pl.jb;
+    pl.nt = ((G * pl.jbq + 15) / 16 * 16) <= 32 ? 32 : 64;
+    // 128-key tiles; about one CTA per SM (a stage ring of 96-128 KB), at
+    // least two tiles per CTA, no CTA with more than 128 tiles.
+    const int tiles_tc = (max_ctx + 127) / 128;
+    const long long units_tc = (long long)B * Hkv * pl.rg;
+    const long long wave_tc = ((long long)num_sms + units_tc - 1) / (units_tc > 0 ? units_tc : 1);
+    const long long len_tc = (tiles_tc + 127) / 128;
+    const long long want_tc = wave_tc > len_tc ? wave_tc : len_tc;
+    int St = 1;
+    while (St < 16 && St < want_tc && (St * 2) * 2 <= tiles_tc) St *= 2;
+    pl.cluster = St;
+    pl.tiles_per_split = (tiles_tc + St - 1) / St;
+    pl.max_splits = St;
+  }
   return pl;
 }
 
@@ -641,6 +670,7 @@ int attn_max_active_clusters(int D, int mt, int wk, int S, int Hkv, int B) {
 
 cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& pl, int* err,
                                cudaStream_t stream) {
+  if (pl.kind == 1) return launch_verify_attn_tc(a, pl, err, stream);
   // Pool as {64 columns, rows, half}: a {64, 16, H} box is one page of one
   // head, both 128-byte halves, landing as [half][16 rows][128 B].
   CUtensorMap maps[4];

@@ -70,6 +70,14 @@ def test_attention_host_validation(lib):
     assert f(ctypes.byref(_dims(batch=0)), 0, *([nul] * 8), nul) == 0
 
 
+def test_attention_plan_host_validation(lib):
+    f = lib.cospec_verify_attn_plan
+    k, sp = ctypes.c_int(), ctypes.c_int()
+    assert f(ctypes.byref(_dims(head_dim=96)), 4096, ctypes.byref(k), ctypes.byref(sp)) == -2
+    assert f(ctypes.byref(_dims()), 4096, None, None) == -1
+    assert f(ctypes.byref(_dims()), 300 * 16 + 1, ctypes.byref(k), ctypes.byref(sp)) == -1
+
+
 def test_lmhead_host_validation(lib):
     f = lib.cospec_lmhead_argmax_features
     assert f(0, 4096, 1000, *([None] * 6), 0, None) == 0          # no rows: nothing to do

@@ -68,6 +68,17 @@ ATTN_CASES = [
     (2, 32, 128, 8, 64, [300, 1500], True),         # 512 rows per KV head: 8 row groups
 ]
 
+# Batches with a (sequence, KV head, row group) per SM and more than 32 query
+# rows per group select the tcgen05 kernel.
+_ctx = lambda n, seed: list(np.random.default_rng(seed).integers(0, 700, n))
+ATTN_TC_CASES = [
+    (24, 8, 64, 8, 128, [0, 1, 63, 64, 65, 127, 128, 129] + _ctx(16, 1), True),  # G = 8: 64 rows
+    (20, 4, 128, 8, 64, _ctx(20, 2), True),         # head_dim 64, G = 16: 64 rows
+    (10, 8, 128, 8, 128, _ctx(10, 3), True),        # 128 rows: two row groups
+    (20, 8, 40, 8, 128, _ctx(20, 4), False),        # G = 5: 40 rows
+    (20, 16, 32, 8, 128, [2000] + _ctx(19, 5), True),  # G = 4, 16 block rows: 64 rows, longer context
+]
+
 
 @pytest.mark.parametrize("case", ATTN_CASES, ids=lambda c: f"B{c[0]}R{c[1]}G{c[2]//c[3]}D{c[4]}")
 def test_verify_attention_matches_oracle(case):
@@ -75,6 +86,7 @@ def test_verify_attention_matches_oracle(case):
     rng = np.random.default_rng(B * 1000 + R * 100 + Hq + D + sum(ctx))
     t = _paged_case(rng, B, R, Hq, Hkv, D, ctx, shuffled)
     max_ctx = max(ctx)
+    assert C.verify_attn_plan(t["q"], t["k_pages"], t["page_table"], max_ctx)[0] == C.ATTN_MMA_SYNC
     out = torch.empty_like(t["q"])
     C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
                   t["ctx_len"], out, max_ctx)
@@ -82,6 +94,28 @@ def test_verify_attention_matches_oracle(case):
                              host(t["v_pages"]), t["table_np"], t["ctx_np"], 16)
     assert_close(host(out), ref, "attention")
     # a second call gives the same bits
+    out2 = torch.empty_like(out)
+    C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
+                  t["ctx_len"], out2, max_ctx)
+    assert torch.equal(out, out2)
+
+
+@pytest.mark.parametrize("case", ATTN_TC_CASES, ids=lambda c: f"B{c[0]}R{c[1]}G{c[2] // c[3]}D{c[4]}")
+def test_verify_attention_tcgen05_matches_oracle(case):
+    B, R, Hq, Hkv, D, ctx, shuffled = case
+    rng = np.random.default_rng(B * 1000 + R * 100 + Hq + D + int(sum(ctx)))
+    t = _paged_case(rng, B, R, Hq, Hkv, D, ctx, shuffled)
+    max_ctx = int(max(ctx))
+    jb = 64 // (Hq // Hkv)
+    if C.num_sms() > B * Hkv * (-(-R // jb)):
+        pytest.skip("more SMs than (sequence, head, row group) units on this device")
+    assert C.verify_attn_plan(t["q"], t["k_pages"], t["page_table"], max_ctx)[0] == C.ATTN_TCGEN05
+    out = torch.empty_like(t["q"])
+    C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
+                  t["ctx_len"], out, max_ctx)
+    ref = O.verify_attention(host(t["q"]), host(t["k_blk"]), host(t["v_blk"]), host(t["k_pages"]),
+                             host(t["v_pages"]), t["table_np"], t["ctx_np"], 16)
+    assert_close(host(out), ref, "attention (tcgen05)")
     out2 = torch.empty_like(out)
     C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
                   t["ctx_len"], out2, max_ctx)
