@@ -481,7 +481,8 @@ def main():
 # (profiles/), keyed by (workload, kernel); an entry is removed when its
 # kernel changes after the capture.
 TRAFFIC = {
-    ("qwen3_8b_b1", "lmhead_argmax_features"): 1247835632.0,
+    ("qwen3_8b_b1", "verify_attn"): 16915200.0,
+    ("qwen3_8b_b1", "lmhead_argmax_features"): 1247979104.0,
 }
 
 
