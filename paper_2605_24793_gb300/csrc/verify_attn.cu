@@ -644,12 +644,13 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
     pl.jbq = jbq;
     pl.rg = (R + pl.jb - 1) / pl.jb;
     pl.nt = ((G * pl.jbq + 15) / 16 * 16) <= 32 ? 32 : 64;
-    // 128-key tiles; about one CTA per SM (a stage ring of 96-128 KB), at
-    // least two tiles per CTA, no CTA with more than 128 tiles.
+    // 128-key tiles; about one CTA per SM (a stage ring of 96-192 KB), at
+    // least two tiles per CTA, no CTA with more than 64 tiles (long
+    // sequences split, so that uneven contexts balance over the waves).
     const int tiles_tc = (max_ctx + 127) / 128;
     const long long units_tc = (long long)B * Hkv * pl.rg;
     const long long wave_tc = ((long long)num_sms + units_tc - 1) / (units_tc > 0 ? units_tc : 1);
-    const long long len_tc = (tiles_tc + 127) / 128;
+    const long long len_tc = (tiles_tc + 63) / 64;
     const long long want_tc = wave_tc > len_tc ? wave_tc : len_tc;
     int St = 1;
     while (St < 16 && St < want_tc && (St * 2) * 2 <= tiles_tc) St *= 2;
