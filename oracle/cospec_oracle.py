@@ -12,7 +12,9 @@ arithmetic below is float64.
 Pins (what fixes each function other than itself; see tests/test_oracle_*.py):
   verify_attention      brute force on tiny inputs, closed forms (two-key
                         3:1 weights, constant V, single visible key), GQA
-                        head mapping, causality, paged == contiguous.
+                        head mapping, causality, paged == contiguous; the
+                        full block mask against the arbitrator's hybrid mask
+                        over a dense sequence (Sec. 3.3).
   lmhead_stats          closed forms (one-hot logits, uniform logits, two
                         classes), tie-break, torch float64 cross-check.
   row_stats_sampled     Philox4x32-10 known-answer vectors of the generator's
@@ -70,17 +72,22 @@ def gather_context(pages, page_table_row, ctx_len: int, page_size: int) -> np.nd
 def verify_attention(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len,
                      page_size: int, scale: Optional[float] = None,
                      seqs: Optional[Sequence[int]] = None,
-                     heads: Optional[Sequence[int]] = None) -> np.ndarray:
-    """Attention of the K+1 block rows of one layer (teacher-forced verify, Eq. 2).
+                     heads: Optional[Sequence[int]] = None,
+                     block_mask: str = "causal") -> np.ndarray:
+    """Attention of the block rows of one layer (teacher-forced verify, Eq. 2).
 
     q [B,R,Hq,D]; k_blk, v_blk [B,R,Hkv,D] (the block's own keys/values);
     k_pages, v_pages [num_pages,Hkv,P,D]; page_table [B,max_pages];
     ctx_len [B].  Block row j of sequence b sits at absolute position C_b + j
     and attends to the C_b committed positions and to block rows 0..j
-    (causal).  Query head h reads KV head floor(h / G), G = Hq / Hkv.
-    Returns o [B,R,Hq,D] float64; rows of sequences / heads not selected by
-    ``seqs`` / ``heads`` are left at zero.
+    (``block_mask="causal"``), or to every block row (``"full"``: the
+    draft/target region of the arbitrator input, Sec. 3.3, which sees the
+    whole context and itself bidirectionally).  Query head h reads KV head
+    floor(h / G), G = Hq / Hkv.  Returns o [B,R,Hq,D] float64; rows of
+    sequences / heads not selected by ``seqs`` / ``heads`` are left at zero.
     """
+    if block_mask not in ("causal", "full"):
+        raise ValueError(block_mask)
     q = _f64(q); k_blk = _f64(k_blk); v_blk = _f64(v_blk)
     k_pages = _f64(k_pages); v_pages = _f64(v_pages)
     page_table = _i64(page_table); ctx_len = _i64(ctx_len)
@@ -95,7 +102,11 @@ def verify_attention(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len,
         keys = np.concatenate([gather_context(k_pages, page_table[b], C, page_size), k_blk[b]], axis=0)
         vals = np.concatenate([gather_context(v_pages, page_table[b], C, page_size), v_blk[b]], axis=0)
         # visible[j, t]: key position t is seen by block row j iff t <= C + j
-        visible = np.arange(C + R)[None, :] <= (C + np.arange(R))[:, None]
+        # (causal), every position (full)
+        if block_mask == "causal":
+            visible = np.arange(C + R)[None, :] <= (C + np.arange(R))[:, None]
+        else:
+            visible = np.ones((R, C + R), dtype=bool)
         for h in (range(Hq) if heads is None else heads):
             kvh = h // G
             s = (q[b, :, h, :] @ keys[:, kvh, :].T) * scale           # [R, C+R]
@@ -105,6 +116,30 @@ def verify_attention(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len,
             p = p / p.sum(axis=1, keepdims=True)
             out[b, :, h, :] = p @ vals[:, kvh, :]
     return out
+
+
+def hybrid_mask(l_c: int, n_region: int) -> np.ndarray:
+    """The arbitrator's attention pattern over q = [c, region] (Sec. 3.3):
+    context positions attend causally within the context; region positions
+    (the draft/target block with its separators) attend to the whole context
+    and to the whole region; no context position attends to the region.
+    Returns visible [l, l] (query, key), l = l_c + n_region."""
+    l = l_c + n_region
+    i = np.arange(l)[:, None]
+    t = np.arange(l)[None, :]
+    return np.where(i < l_c, t <= i, True)
+
+
+def dense_masked_attention(q, k, v, visible, scale: Optional[float] = None) -> np.ndarray:
+    """softmax(q k^T * scale, masked) v for one head over a dense sequence:
+    q, k, v [l, D], visible [l, l] boolean.  float64."""
+    q = _f64(q); k = _f64(k); v = _f64(v)
+    if scale is None:
+        scale = 1.0 / math.sqrt(q.shape[1])
+    s = np.where(visible, (q @ k.T) * scale, -np.inf)
+    s = s - s.max(axis=1, keepdims=True)
+    p = np.exp(s)
+    return (p / p.sum(axis=1, keepdims=True)) @ v
 
 
 # ---------------------------------------------------------------------------

@@ -147,3 +147,81 @@ def test_selected_rows_only():
     part = O.verify_attention(q, kb, vb, kp, vp, table, np.array(ctx), P, seqs=[1], heads=[3])
     np.testing.assert_array_equal(part[1, :, 3], full[1, :, 3])
     assert not part[0].any() and not part[2].any()
+
+
+# --- the arbitrator's hybrid mask (Sec. 3.3): region rows see the context and
+# --- the whole region; the context never sees the region
+
+def test_hybrid_mask_shape_and_rules():
+    m = O.hybrid_mask(3, 4)
+    assert m.shape == (7, 7)
+    # context rows: causal, never the region
+    for i in range(3):
+        assert list(m[i]) == [t <= i for t in range(7)]
+    # region rows: everything
+    assert m[3:].all()
+
+
+def test_full_block_mask_equals_dense_hybrid_attention():
+    """The region rows of the dense hybrid-masked attention equal the paged
+    block attention with the full block mask: context as the cache, region as
+    the block."""
+    rng = np.random.default_rng(11)
+    l_c, n, Hq, Hkv, D, P = 13, 7, 4, 2, 8, 4
+    q = rng.standard_normal((l_c + n, Hq, D)) * 1.5
+    k = rng.standard_normal((l_c + n, Hkv, D))
+    v = rng.standard_normal((l_c + n, Hkv, D))
+    mask = O.hybrid_mask(l_c, n)
+    dense = np.stack([O.dense_masked_attention(q[:, h], k[:, h // 2], v[:, h // 2], mask)
+                      for h in range(Hq)], axis=1)                      # [l, Hq, D]
+    # the same tokens as one sequence: context in pages, region as the block
+    npages = (l_c + n + P - 1) // P
+    kp = np.zeros((npages, Hkv, P, D)); vp = np.zeros((npages, Hkv, P, D))
+    for t in range(l_c):
+        kp[t // P, :, t % P] = k[t]; vp[t // P, :, t % P] = v[t]
+    table = np.arange(npages)[None, :]
+    got = O.verify_attention(q[None, l_c:], k[None, l_c:], v[None, l_c:], kp, vp, table,
+                             np.array([l_c]), P, block_mask="full")
+    np.testing.assert_allclose(got[0], dense[l_c:], rtol=1e-12, atol=1e-12)
+    # and the context rows of the dense pass are plain causal attention over the context
+    causal = np.stack([O.dense_masked_attention(q[:l_c, h], k[:l_c, h // 2], v[:l_c, h // 2],
+                                                np.tril(np.ones((l_c, l_c), dtype=bool)))
+                       for h in range(Hq)], axis=1)
+    np.testing.assert_allclose(dense[:l_c], causal, rtol=1e-12, atol=1e-12)
+
+
+def test_full_and_causal_block_agree_on_the_last_row_only():
+    rng = np.random.default_rng(12)
+    B, R, Hq, Hkv, D, P = 2, 5, 4, 2, 8, 4
+    ctx = [9, 0]
+    kp, vp, table = _contiguous_pages(ctx, R, Hkv, P, D, rng)
+    q = rng.standard_normal((B, R, Hq, D)) * 2
+    kb = rng.standard_normal((B, R, Hkv, D)); vb = rng.standard_normal((B, R, Hkv, D))
+    full = O.verify_attention(q, kb, vb, kp, vp, table, np.array(ctx), P, block_mask="full")
+    causal = O.verify_attention(q, kb, vb, kp, vp, table, np.array(ctx), P)
+    np.testing.assert_allclose(full[:, R - 1], causal[:, R - 1], rtol=1e-12, atol=1e-12)
+    assert np.abs(full[:, 0] - causal[:, 0]).max() > 1e-3
+
+
+def test_full_block_brute_force():
+    rng = np.random.default_rng(13)
+    B, R, Hq, Hkv, D, P = 2, 3, 4, 2, 4, 4
+    ctx = [5, 2]
+    kp, vp, table = _contiguous_pages(ctx, R, Hkv, P, D, rng)
+    q = rng.standard_normal((B, R, Hq, D)) * 2
+    kb = rng.standard_normal((B, R, Hkv, D)); vb = rng.standard_normal((B, R, Hkv, D))
+    got = O.verify_attention(q, kb, vb, kp, vp, table, np.array(ctx), P, block_mask="full")
+    G = Hq // Hkv
+    for b in range(B):
+        for j in range(R):
+            for h in range(Hq):
+                keys, vals = [], []
+                for t in range(ctx[b]):
+                    keys.append(kp[table[b][t // P], h // G, t % P]); vals.append(vp[table[b][t // P], h // G, t % P])
+                for jj in range(R):                     # every block row, before or after j
+                    keys.append(kb[b, jj, h // G]); vals.append(vb[b, jj, h // G])
+                sc = [sum(qe * ke for qe, ke in zip(q[b, j, h], kk)) / math.sqrt(D) for kk in keys]
+                mx = max(sc)
+                w = [math.exp(x - mx) for x in sc]
+                ref = [sum(wi * vv[e] for wi, vv in zip(w, vals)) / sum(w) for e in range(D)]
+                np.testing.assert_allclose(got[b, j, h], ref, rtol=1e-12, atol=1e-12)
