@@ -103,7 +103,7 @@ COSPEC_API int cospec_num_sms(void);
  *    mma.sync tensor-core tiles, and one on tcgen05 (TMEM accumulators),
  *    used when a KV head's group has more than 32 query rows and the batch
  *    gives every SM a (sequence, KV head, row group) of its own.
- *    Supported: head_dim in {64, 128}; page_size == 16; rows <= 32;
+ *    Supported: head_dim in {64, 128}; page_size == 16; rows <= 64;
  *    num_q_heads % num_kv_heads == 0; (num_q_heads / num_kv_heads) * rows <= 512.
  * ------------------------------------------------------------------------ */
 typedef struct {
@@ -124,6 +124,14 @@ typedef struct {
  * when that kernel writes none of them (e.g. between the layers of one
  * round, where only q / k_blk / v_blk come from the previous layer). */
 #define COSPEC_ATTN_KV_STABLE 1
+
+/* Every block row attends to every block row instead of rows 0..j only: the
+ * draft/target region of the arbitrator's input (Sec. 3.3), which sees the
+ * whole context causally cached before it and itself bidirectionally, the
+ * context never seeing the region.  With the region's 2K+3 tokens as the
+ * block (rows <= 64, i.e. K <= 30) this is the arbitrator LM's attention
+ * for one round. */
+#define COSPEC_ATTN_BLOCK_FULL 2
 
 /* Launch plan cospec_verify_attn would use for these dimensions on the
  * current device: *kernel = 0 (mma.sync) or 1 (tcgen05), *splits = CTAs per

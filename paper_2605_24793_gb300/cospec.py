@@ -34,6 +34,7 @@ class AttnDims(ctypes.Structure):
 
 
 ATTN_KV_STABLE = 1
+ATTN_BLOCK_FULL = 2
 
 
 class CospecError(RuntimeError):
@@ -131,16 +132,20 @@ def verify_attn_plan(q, k_pages, page_table, max_ctx: int):
 
 
 def verify_attn(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len, out, max_ctx,
-                softmax_scale: float = 0.0, stream=None, kv_stable: bool = False) -> torch.Tensor:
+                softmax_scale: float = 0.0, stream=None, kv_stable: bool = False,
+                block_full: bool = False) -> torch.Tensor:
     """Verify attention of one layer (Sec. 3.1, Eq. 2).  See include/cospec.h.
     ``kv_stable``: the kernel queued just before writes neither ctx_len, the
-    page table nor the cached pages (COSPEC_ATTN_KV_STABLE)."""
+    page table nor the cached pages (COSPEC_ATTN_KV_STABLE).  ``block_full``:
+    block rows see the whole block (the arbitrator's draft/target region,
+    Sec. 3.3; COSPEC_ATTN_BLOCK_FULL)."""
     for t, n in ((q, "q"), (k_blk, "k_blk"), (v_blk, "v_blk"), (k_pages, "k_pages"),
                  (v_pages, "v_pages"), (out, "out")):
         _req(t, torch.bfloat16, n)
     _req(page_table, torch.int32, "page_table", 2)
     _req(ctx_len, torch.int32, "ctx_len", 1)
-    dims = attn_dims(q, k_pages, page_table, softmax_scale, ATTN_KV_STABLE if kv_stable else 0)
+    dims = attn_dims(q, k_pages, page_table, softmax_scale,
+                     (ATTN_KV_STABLE if kv_stable else 0) | (ATTN_BLOCK_FULL if block_full else 0))
     if tuple(k_blk.shape) != (dims.batch, dims.rows, dims.num_kv_heads, dims.head_dim):
         raise ValueError("k_blk shape does not match q / pages")
     if out.shape != q.shape:

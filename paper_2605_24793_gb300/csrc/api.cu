@@ -130,17 +130,19 @@ static int check_attn_dims(const cospec_attn_dims* d) {
     return COSPEC_ERR_INVALID_ARG;
   if (d->num_q_heads % d->num_kv_heads != 0) return COSPEC_ERR_INVALID_ARG;
   if (isnan(d->softmax_scale) || isinf(d->softmax_scale)) return COSPEC_ERR_INVALID_ARG;
-  if (d->flags & ~COSPEC_ATTN_KV_STABLE) return COSPEC_ERR_INVALID_ARG;
+  if (d->flags & ~(COSPEC_ATTN_KV_STABLE | COSPEC_ATTN_BLOCK_FULL)) return COSPEC_ERR_INVALID_ARG;
   if (d->head_dim != 64 && d->head_dim != 128) return COSPEC_ERR_UNSUPPORTED;
   if (d->page_size != 16) return COSPEC_ERR_UNSUPPORTED;
-  if (d->rows > 32) return COSPEC_ERR_UNSUPPORTED;
+  if (d->rows > 64) return COSPEC_ERR_UNSUPPORTED;
   if ((d->num_q_heads / d->num_kv_heads) * d->rows > 512) return COSPEC_ERR_UNSUPPORTED;
   return COSPEC_OK;
 }
 
 // Largest schedulable cluster not above `S` for this variant (cached per device).
-static int schedulable_cluster(int D, const AttnPlan& pl, int Hkv, int B) {
-  static int cache[64][2][6][5];   // [dev][D==128][variant][log2 S] : 0 unknown, 1 ok, -1 no
+static int schedulable_cluster(int D, const AttnPlan& pl, int Hkv, int B, int R) {
+  // [dev][D==128][variant][block keys / 16 - 1][log2 S] : 0 unknown, 1 ok, -1 no
+  static int cache[64][2][6][4][5];
+  const int kbr = (R + 15) & ~15;
   int dev = 0;
   cudaGetDevice(&dev);
   const int di = D == 128 ? 1 : 0;
@@ -150,10 +152,10 @@ static int schedulable_cluster(int D, const AttnPlan& pl, int Hkv, int B) {
   while (S > 1) {
     int ls = 0;
     while ((1 << ls) < S) ++ls;
-    int& c = cache[dev < 64 ? dev : 63][di][mi][ls];
+    int& c = cache[dev < 64 ? dev : 63][di][mi][kbr / 16 - 1][ls];
     if (c == 0)
       c = (pl.kind == 1 ? attn_tc_max_active_clusters(D, pl.nt, S, Hkv, B, pl.rg)
-                        : attn_max_active_clusters(D, pl.mt, pl.wk, S, Hkv, B)) > 0 ? 1 : -1;
+                        : attn_max_active_clusters(D, pl.mt, pl.wk, S, Hkv, B, kbr)) > 0 ? 1 : -1;
     if (c > 0) break;
     S >>= 1;
   }
@@ -170,7 +172,7 @@ COSPEC_API int cospec_verify_attn_plan(const cospec_attn_dims* d, int max_ctx, i
   if (sms <= 0) return COSPEC_ERR_CUDA;
   AttnPlan pl = plan_verify_attn(d->batch, d->rows, d->num_q_heads, d->num_kv_heads,
                                  d->head_dim, max_ctx, sms);
-  pl.cluster = schedulable_cluster(d->head_dim, pl, d->num_kv_heads, d->batch);
+  pl.cluster = schedulable_cluster(d->head_dim, pl, d->num_kv_heads, d->batch, d->rows);
   *kernel = pl.kind;
   *splits = pl.cluster;
   return COSPEC_OK;
@@ -192,7 +194,7 @@ COSPEC_API int cospec_verify_attn(const cospec_attn_dims* d, int max_ctx, const 
   if (sms <= 0) return COSPEC_ERR_CUDA;
   AttnPlan pl = plan_verify_attn(d->batch, d->rows, d->num_q_heads, d->num_kv_heads,
                                  d->head_dim, max_ctx, sms);
-  pl.cluster = schedulable_cluster(d->head_dim, pl, d->num_kv_heads, d->batch);
+  pl.cluster = schedulable_cluster(d->head_dim, pl, d->num_kv_heads, d->batch, d->rows);
   int* err = device_error_word();
   if (!err) return COSPEC_ERR_CUDA;
   AttnArgs a{};
@@ -215,6 +217,7 @@ COSPEC_API int cospec_verify_attn(const cospec_attn_dims* d, int max_ctx, const 
   a.scale = d->softmax_scale > 0.f ? d->softmax_scale : 1.0f / sqrtf((float)d->head_dim);
   a.max_ctx = max_ctx;
   a.kv_stable = (d->flags & COSPEC_ATTN_KV_STABLE) ? 1 : 0;
+  a.block_full = (d->flags & COSPEC_ATTN_BLOCK_FULL) ? 1 : 0;
   return from_cuda(launch_verify_attn(a, pl, err, static_cast<cudaStream_t>(stream)));
 }
 

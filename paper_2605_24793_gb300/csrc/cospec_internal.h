@@ -51,6 +51,7 @@ struct AttnArgs {
   float scale;
   int max_ctx;
   int kv_stable;   // cache-side reads may start before the previous kernel finishes
+  int block_full;  // block rows attend to every block row
 };
 struct AttnPlan {
   int kind;               // 0: mma.sync kernel, 1: tcgen05 kernel
@@ -62,7 +63,7 @@ struct AttnPlan {
   size_t total_bytes;     // workspace (none)
 };
 AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int num_sms);
-int attn_max_active_clusters(int D, int mt, int wk, int S, int Hkv, int B);
+int attn_max_active_clusters(int D, int mt, int wk, int S, int Hkv, int B, int kbr);
 cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& plan, int* err,
                                cudaStream_t stream);
 bool tc_attn_supported(int D, int G);

@@ -40,6 +40,7 @@ struct AttnParams {
   int max_pages, num_pages;
   float scale_log2;
   int kv_stable;
+  int block_full;  // block rows see every block row (not only rows <= their own)
   int* err;
 };
 
@@ -65,7 +66,7 @@ struct Layout {
   static_assert(RECV_END <= NSTAGE * STAGE, "partials must fit in the stage ring");
   static constexpr int BAR = NSTAGE * STAGE;       // full[NSTAGE], empty[NSTAGE], block
   static constexpr int BLK = BAR + (2 * NSTAGE + 2) * 8 + 1024;   // 1024-aligned block K/V
-  // the block region holds 2*H halves of KBR rows (KBR = 16 or 32, runtime)
+  // the block region holds 2*H halves of KBR rows (KBR = 16, 32, 48 or 64, runtime)
   static constexpr int blk_half(int kbr) { return kbr * ROWB; }
   static constexpr int total(int kbr) { return BLK / 1024 * 1024 + 2 * H * kbr * ROWB; }
 };
@@ -379,12 +380,13 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
       }
       named_bar_sync(1, NTC);
       if (wk == 0) {
-        if (KBR == 16)
-          attend<D, 16>(smem_u32(blk_k), smem_u32(blk_v), PAGE * ROWB, 16 * ROWB, 0, 0, true, j0,
-                        j1, p.scale_log2, qf, o, m0, m1, l0, l1, lane);
-        else
-          attend<D, 32>(smem_u32(blk_k), smem_u32(blk_v), PAGE * ROWB, 32 * ROWB, 0, 0, true, j0,
-                        j1, p.scale_log2, qf, o, m0, m1, l0, l1, lane);
+        // causal: block key j is seen by the rows of block rows >= j; full: by every row
+        const int b0 = p.block_full ? p.R - 1 : j0, b1 = p.block_full ? p.R - 1 : j1;
+        const uint32_t sk = smem_u32(blk_k), sv = smem_u32(blk_v);
+        // 16 block keys at a time (one code path for any block length)
+        for (int g0 = 0; g0 < KBR; g0 += 16)
+          attend<D, 16>(sk, sv, PAGE * ROWB, KBR * ROWB, g0, g0, true, b0, b1, p.scale_log2, qf, o,
+                        m0, m1, l0, l1, lane);
       }
     }
     // After a timed-out wait a copy may still be in flight: wait (bounded)
@@ -540,18 +542,23 @@ template <int D, int MT, int WK>
 cudaError_t launch_t(const CUtensorMap* maps, const AttnParams& p, int S, int B, int Hkv,
                      cudaStream_t stream) {
   using LY = Layout<D, MT, WK>;
-  const size_t smem = LY::total(p.R <= 16 ? 16 : 32) + 1024;
-  static bool configured[64] = {false};
+  const size_t smem = LY::total((p.R + 15) & ~15) + 1024;
+  // The dynamic shared-memory limit only grows (to what the largest launch
+  // so far needs), so graphs captured earlier stay launchable.
+  static size_t configured[64] = {0};
+  static bool cluster_ok[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
   auto kern = verify_attn_kernel<D, MT, WK>;
-  if (dev < 64 && !configured[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)(LY::total(32) + 1024));
+  if (dev < 64 && configured[dev] < smem) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    configured[dev] = smem;
+  }
+  if (dev < 64 && !cluster_ok[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
-    configured[dev] = true;
+    cluster_ok[dev] = true;
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(S, Hkv * p.RG, B);
@@ -571,15 +578,21 @@ cudaError_t launch_t(const CUtensorMap* maps, const AttnParams& p, int S, int B,
 }
 
 template <int D, int MT, int WK>
-int max_cluster_t(int S, int Hkv, int B) {
+int max_cluster_t(int S, int Hkv, int B, int kbr) {
   using LY = Layout<D, MT, WK>;
   auto kern = verify_attn_kernel<D, MT, WK>;
-  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(LY::total(32) + 1024));
+  // the occupancy query needs the limit at least at the queried size; it
+  // never lowers a limit a launch has raised
+  int cur = 0;
+  cudaFuncAttributes fa;
+  if (cudaFuncGetAttributes(&fa, kern) == cudaSuccess) cur = fa.maxDynamicSharedSizeBytes;
+  if (cur < (int)(LY::total(kbr) + 1024))
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(LY::total(kbr) + 1024));
   cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(S, Hkv, B);
   cfg.blockDim = dim3(MT * WK * 32 + 32, 1, 1);
-  cfg.dynamicSmemBytes = LY::total(16) + 1024;
+  cfg.dynamicSmemBytes = LY::total(kbr) + 1024;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = S;
@@ -661,9 +674,9 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
   return pl;
 }
 
-int attn_max_active_clusters(int D, int mt, int wk, int S, int Hkv, int B) {
+int attn_max_active_clusters(int D, int mt, int wk, int S, int Hkv, int B, int kbr) {
 #define X(DD, MM, WW) \
-  if (D == DD && mt == MM && wk == WW) return max_cluster_t<DD, MM, WW>(S, Hkv, B);
+  if (D == DD && mt == MM && wk == WW) return max_cluster_t<DD, MM, WW>(S, Hkv, B, kbr);
   COSPEC_ATTN_VARIANTS(X)
 #undef X
   return 0;
@@ -683,7 +696,7 @@ cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& pl, int* err,
   // Block K/V as {64 columns, batch*rows, half, head}: one box per (b, head).
   const uint64_t db[4] = {64, (uint64_t)a.B * a.R, (uint64_t)H, (uint64_t)a.Hkv};
   const uint64_t sb[3] = {(uint64_t)a.Hkv * a.D * 2, 128, (uint64_t)a.D * 2};
-  const uint32_t bb[4] = {64, (uint32_t)(a.R <= 16 ? 16 : 32), (uint32_t)H, 1};
+  const uint32_t bb[4] = {64, (uint32_t)((a.R + 15) & ~15), (uint32_t)H, 1};
   if (!encode_tensor_map_bf16(&maps[0], a.k_pages, 3, dp, sp, bp) ||
       !encode_tensor_map_bf16(&maps[1], a.v_pages, 3, dp, sp, bp) ||
       !encode_tensor_map_bf16(&maps[2], a.k_blk, 4, db, sb, bb) ||
@@ -705,6 +718,7 @@ cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& pl, int* err,
   p.num_pages = a.num_pages;
   p.scale_log2 = a.scale * 1.4426950408889634f;
   p.kv_stable = a.kv_stable;
+  p.block_full = a.block_full;
   p.err = err;
 #define X(DD, MM, WW)                                      \
   if (a.D == DD && pl.mt == MM && pl.wk == WW)             \

@@ -57,6 +57,7 @@ struct TcParams {
   int max_pages, num_pages;
   float scale_log2;
   int kv_stable;
+  int block_full;  // block rows see every block row (not only rows <= their own)
   int* err;
 };
 
@@ -460,7 +461,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       // rows of block rows >= j (causal inside the block)
       const bool kvalid = blk ? (key < p.R) : ((t_begin + t) * TKT + key < C);
       // block key j is seen by row r iff j <= j0 + r / G, i.e. (j - j0) * G <= r
-      const int kg = (key - j0) * p.G;
+      // (causal), or by every row (full block)
+      const int kg = p.block_full ? -1 : (key - j0) * p.G;
       float x[NT];
       float excess = -INFINITY;
       if (s_warp && okw) {
@@ -849,6 +851,7 @@ cudaError_t launch_verify_attn_tc(const AttnArgs& a, const AttnPlan& pl, int* er
   p.num_pages = a.num_pages;
   p.scale_log2 = a.scale * 1.4426950408889634f;
   p.kv_stable = a.kv_stable;
+  p.block_full = a.block_full;
   p.err = err;
   if (a.D == 128 && pl.nt == 32) return launch_tc_t<128, 32>(maps, p, pl.cluster, a.B, a.Hkv, pl.rg, stream);
   if (a.D == 128 && pl.nt == 64) return launch_tc_t<128, 64>(maps, p, pl.cluster, a.B, a.Hkv, pl.rg, stream);

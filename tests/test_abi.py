@@ -61,11 +61,13 @@ def test_attention_host_validation(lib):
     # shapes the kernels do not cover
     assert f(ctypes.byref(_dims(head_dim=96)), 4096, *([nul] * 8), nul) == -2
     assert f(ctypes.byref(_dims(page_size=32)), 4096, *([nul] * 8), nul) == -2
-    assert f(ctypes.byref(_dims(rows=33)), 4096, *([nul] * 8), nul) == -2
+    assert f(ctypes.byref(_dims(rows=65)), 4096, *([nul] * 8), nul) == -2
     assert f(ctypes.byref(_dims(num_q_heads=30)), 4096, *([nul] * 8), nul) == -1
     assert f(ctypes.byref(_dims(softmax_scale=float("nan"))), 4096, *([nul] * 8), nul) == -1
     # max_ctx beyond the page-table row
     assert f(ctypes.byref(_dims()), 300 * 16 + 1, *([nul] * 8), nul) == -1
+    # unknown flag bits
+    assert f(ctypes.byref(_dims(flags=4)), 4096, *([nul] * 8), nul) == -1
     # empty batch is a no-op
     assert f(ctypes.byref(_dims(batch=0)), 0, *([nul] * 8), nul) == 0
 

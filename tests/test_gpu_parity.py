@@ -122,6 +122,42 @@ def test_verify_attention_tcgen05_matches_oracle(case):
     assert torch.equal(out, out2)
 
 
+# The arbitrator's draft/target region (Sec. 3.3): 2K+3 block rows that see
+# the whole block; K = 7 gives 17 rows, K = 25 (the paper's default) 53.
+ATTN_FULL_CASES = [
+    # B, R, Hq, Hkv, D, contexts, shuffled, expected kernel
+    (1, 17, 32, 8, 128, [4096], False, 0),          # K = 7 region on a Qwen3-4B-like arbitrator
+    (3, 53, 32, 8, 128, [0, 300, 2500], True, 0),   # K = 25 region: 53 rows, 4 block-key groups of 16
+    (2, 9, 16, 8, 64, [100, 33], True, 0),          # head_dim 64, K = 3 region
+    (20, 53, 8, 8, 128, _ctx(20, 6), True, 1),      # G = 1, 53 rows per group: tcgen05 kernel
+    (24, 17, 32, 8, 128, _ctx(24, 7), True, 1),     # G = 4, 64-row groups: tcgen05 kernel
+]
+
+
+@pytest.mark.parametrize("case", ATTN_FULL_CASES, ids=lambda c: f"B{c[0]}R{c[1]}G{c[2] // c[3]}D{c[4]}")
+def test_verify_attention_full_block_matches_oracle(case):
+    B, R, Hq, Hkv, D, ctx, shuffled, kernel = case
+    rng = np.random.default_rng(B * 1000 + R * 100 + Hq + D + int(sum(ctx)) + 77)
+    t = _paged_case(rng, B, R, Hq, Hkv, D, ctx, shuffled)
+    max_ctx = int(max(ctx))
+    jb = 64 // (Hq // Hkv)
+    if kernel == 1 and C.num_sms() > B * Hkv * (-(-R // jb)):
+        pytest.skip("more SMs than (sequence, head, row group) units on this device")
+    assert C.verify_attn_plan(t["q"], t["k_pages"], t["page_table"], max_ctx)[0] == kernel
+    out = torch.empty_like(t["q"])
+    C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
+                  t["ctx_len"], out, max_ctx, block_full=True)
+    ref = O.verify_attention(host(t["q"]), host(t["k_blk"]), host(t["v_blk"]), host(t["k_pages"]),
+                             host(t["v_pages"]), t["table_np"], t["ctx_np"], 16, block_mask="full")
+    assert_close(host(out), ref, "attention (full block)")
+    # the causal call on the same inputs still matches the causal oracle
+    C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
+                  t["ctx_len"], out, max_ctx)
+    ref_c = O.verify_attention(host(t["q"]), host(t["k_blk"]), host(t["v_blk"]), host(t["k_pages"]),
+                               host(t["v_pages"]), t["table_np"], t["ctx_np"], 16)
+    assert_close(host(out), ref_c, "attention (causal, long block)")
+
+
 def test_verify_attention_split_count_does_not_change_result_beyond_tolerance():
     rng = np.random.default_rng(3)
     t = _paged_case(rng, 2, 6, 32, 8, 128, [3000, 5000], True)
