@@ -63,6 +63,8 @@ typedef enum {
                                     accepted rows > max_pages_per_seq * page_size (commit) */
 #define COSPEC_DEVERR_TOKEN 4    /* token id outside the vocabulary */
 #define COSPEC_DEVERR_TIMEOUT 8  /* a bounded pipeline wait gave up (never expected) */
+#define COSPEC_DEVERR_OFFSETS 16 /* a group / round offset array is not non-decreasing within
+                                    its range (RL call); the group is skipped */
 
 /* Human-readable name of a cospec_status value (static string). */
 COSPEC_API const char* cospec_status_string(int status);
@@ -275,6 +277,60 @@ COSPEC_API int cospec_accept_commit(int B, int K, int num_layers, const cospec_a
                                     const uint16_t* v_blk, uint16_t* k_pages, uint16_t* v_pages,
                                     long long pool_layer_stride, const int32_t* page_table,
                                     int32_t* ctx_len, int32_t* accept_len, int32_t* emitted,
+                                    void* stream);
+
+/* ------------------------------------------------------------------------ */
+/* 5. RL stage: reward shaping, returns and advantages (Sec. 3.4).
+ *
+ *    A batch of prompt groups: group x owns rollouts group_off[x] ..
+ *    group_off[x+1]-1, rollout m owns rounds round_off[m] .. round_off[m+1]-1,
+ *    and round r holds K draft positions (index i-1 for position i): match
+ *    (Delta_i, Eq. 3), accept (a_i; ignored at matches) and ell
+ *    (log p_T(y_hat_i | ...), Eq. 23).  Per round: s = first rejected
+ *    mismatch else K+1, i* = first mismatch, rho = (s - i*) / (K+1 - i*), the
+ *    effective decisions I_r = mismatches at positions <= min(s, K).
+ *      g      correct rollout: rho; incorrect: -alpha |ell_i| for accepted
+ *             mismatches before the first rejection, -beta at the rejection
+ *      J[m]   sum of g over the rollout's effective decisions
+ *      Jbar   J, with the correct rollouts of a mixed group scaled by
+ *             gamma = sum_incorrect |J| / (sum_correct J + eps)
+ *      adv[m] eta (Jbar - mu) / (sigma + eps) over the group (population
+ *             sigma; eta = eta_fail for all-incorrect groups, else 1)
+ *      adv_dec  correct: rho * adv[m]; incorrect: |g| / sum |g| * adv[m]
+ *    With ratio, p_new, p_ref (pi_theta / pi_old for the taken action,
+ *    pi_theta(a=1), pi_ref(a=1) per decision) also the objective:
+ *      loss[0] = sum min(ratio A, clip(ratio, 1 -+ clip_eps) A), loss[1] =
+ *      sum Bernoulli entropy of p_new, loss[2] = sum KL(p_new || p_ref) over
+ *      the effective decisions, loss[3] = -loss[0] - beta_h loss[1] + beta_kl loss[2].
+ *
+ *    group_off int32 [num_groups+1]; correct uint8 [num_rollouts];
+ *    round_off int32 [num_rollouts+1]; match, accept uint8 [num_rounds, K];
+ *    ell float32 [num_rounds, K]; 1 <= K <= 64.
+ *    Outputs (float32): g, adv_dec [num_rounds, K] (0 outside effective
+ *    decisions), eff uint8 [num_rounds, K], rho [num_rounds] (NaN without a
+ *    mismatch), J, Jbar, adv [num_rollouts]; loss [4] (only when ratio,
+ *    p_new and p_ref are given; all three or none).  Group statistics are
+ *    computed in float64.  ws >= cospec_rl_workspace(...) bytes.
+ * ------------------------------------------------------------------------ */
+typedef struct {
+  float alpha;     /* risk penalty weight (the paper: 1.0) */
+  float beta;      /* rejection penalty (0.25) */
+  float eta_fail;  /* weight of all-incorrect groups (0.5) */
+  float eps;       /* normaliser epsilon, > 0 */
+  float clip_eps;  /* PPO clip range (0.2) */
+  float beta_h;    /* entropy coefficient (0.01) */
+  float beta_kl;   /* KL coefficient (0.02) */
+} cospec_rl_params;
+
+COSPEC_API size_t cospec_rl_workspace(int num_groups, int num_rollouts);
+COSPEC_API int cospec_rl_advantages(int num_groups, int num_rollouts, int num_rounds, int K,
+                                    const int32_t* group_off, const uint8_t* correct,
+                                    const int32_t* round_off, const uint8_t* match,
+                                    const uint8_t* accept, const float* ell,
+                                    const cospec_rl_params* params, const float* ratio,
+                                    const float* p_new, const float* p_ref, float* g,
+                                    uint8_t* eff, float* rho, float* J, float* Jbar, float* adv,
+                                    float* adv_dec, float* loss, void* ws, size_t ws_bytes,
                                     void* stream);
 
 #ifdef __cplusplus

@@ -17,12 +17,13 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libcospec.so")
 
 POLICY_MLP, POLICY_TARGET, POLICY_DRAFT = 0, 1, 2
-DEVERR_PAGE, DEVERR_CTX, DEVERR_TOKEN, DEVERR_TIMEOUT = 1, 2, 4, 8
+DEVERR_PAGE, DEVERR_CTX, DEVERR_TOKEN, DEVERR_TIMEOUT, DEVERR_OFFSETS = 1, 2, 4, 8, 16
 
 EXPORTED = ("cospec_status_string", "cospec_get_device_error", "cospec_num_sms",
             "cospec_verify_attn", "cospec_lmhead_workspace", "cospec_lmhead_argmax_features",
             "cospec_arbitrate", "cospec_accept_commit", "cospec_lmhead_argmax_features_noalloc",
-            "cospec_lmhead_sample_features", "cospec_verify_attn_plan")
+            "cospec_lmhead_sample_features", "cospec_verify_attn_plan", "cospec_rl_workspace",
+            "cospec_rl_advantages")
 
 
 class AttnDims(ctypes.Structure):
@@ -31,6 +32,16 @@ class AttnDims(ctypes.Structure):
                 ("page_size", ctypes.c_int), ("max_pages_per_seq", ctypes.c_int),
                 ("num_pages", ctypes.c_int), ("softmax_scale", ctypes.c_float),
                 ("flags", ctypes.c_int)]
+
+
+class RLParams(ctypes.Structure):
+    """cospec_rl_params; defaults are the paper's (App. C)."""
+    _fields_ = [(n, ctypes.c_float) for n in
+                ("alpha", "beta", "eta_fail", "eps", "clip_eps", "beta_h", "beta_kl")]
+
+    def __init__(self, alpha=1.0, beta=0.25, eta_fail=0.5, eps=1e-6, clip_eps=0.2, beta_h=0.01,
+                 beta_kl=0.02):
+        super().__init__(alpha, beta, eta_fail, eps, clip_eps, beta_h, beta_kl)
 
 
 ATTN_KV_STABLE = 1
@@ -61,6 +72,10 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "cospec_num_sms": (_i, []),
         "cospec_verify_attn": (_i, [_PDIMS, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
         "cospec_verify_attn_plan": (_i, [_PDIMS, _i, ctypes.POINTER(_i), ctypes.POINTER(_i)]),
+        "cospec_rl_workspace": (_sz, [_i, _i]),
+        "cospec_rl_advantages": (_i, [_i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp,
+                                      ctypes.POINTER(RLParams), _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                      _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
         "cospec_lmhead_workspace": (_sz, [_i, _i, _i]),
         "cospec_lmhead_argmax_features": (_i, [_i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
         "cospec_lmhead_argmax_features_noalloc": (_i, [_i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp]),
@@ -225,6 +240,49 @@ def lmhead_argmax_features_noalloc(hidden, w, draft_for_row, argmax, stats, stre
         M, d, V, _ptr(hidden), _ptr(w), _ptr(draft_for_row), _ptr(argmax), _ptr(stats),
         _stream(stream)))
     return argmax, stats
+
+
+def rl_advantages(group_off, correct, round_off, match, accept, ell, params: RLParams = None,
+                  ratio=None, p_new=None, p_ref=None, stream=None) -> dict:
+    """RL-stage rewards and advantages (Sec. 3.4).  Inputs are CUDA tensors:
+    group_off int32 [G+1], correct uint8 [M], round_off int32 [M+1],
+    match / accept uint8 [R, K], ell float32 [R, K]; optional ratio / p_new /
+    p_ref float32 [R, K] for the objective.  Returns the output tensors."""
+    params = params if params is not None else RLParams()
+    _req(group_off, torch.int32, "group_off", 1)
+    _req(round_off, torch.int32, "round_off", 1)
+    _req(correct, torch.uint8, "correct", 1)
+    _req(match, torch.uint8, "match", 2)
+    _req(accept, torch.uint8, "accept", 2)
+    _req(ell, torch.float32, "ell", 2)
+    G, M = group_off.numel() - 1, correct.numel()
+    R, K = match.shape
+    if round_off.numel() != M + 1 or tuple(accept.shape) != (R, K) or tuple(ell.shape) != (R, K):
+        raise ValueError("inconsistent RL shapes")
+    obj = [t for t in (ratio, p_new, p_ref) if t is not None]
+    for t, n in zip(obj, ("ratio", "p_new", "p_ref")):
+        _req(t, torch.float32, n, 2)
+        if tuple(t.shape) != (R, K):
+            raise ValueError(f"{n} must be [R, K]")
+    dev = match.device
+    out = dict(g=torch.empty((R, K), dtype=torch.float32, device=dev),
+               eff=torch.empty((R, K), dtype=torch.uint8, device=dev),
+               rho=torch.empty(R, dtype=torch.float32, device=dev),
+               J=torch.empty(M, dtype=torch.float32, device=dev),
+               Jbar=torch.empty(M, dtype=torch.float32, device=dev),
+               adv=torch.empty(M, dtype=torch.float32, device=dev),
+               adv_dec=torch.empty((R, K), dtype=torch.float32, device=dev))
+    loss = torch.empty(4, dtype=torch.float32, device=dev) if obj else None
+    lib = load_library()
+    ws = torch.empty(lib.cospec_rl_workspace(G, M), dtype=torch.uint8, device=dev)
+    _check(lib.cospec_rl_advantages(
+        G, M, R, K, _ptr(group_off), _ptr(correct), _ptr(round_off), _ptr(match), _ptr(accept),
+        _ptr(ell), ctypes.byref(params), _ptr(ratio), _ptr(p_new), _ptr(p_ref), _ptr(out["g"]),
+        _ptr(out["eff"]), _ptr(out["rho"]), _ptr(out["J"]), _ptr(out["Jbar"]), _ptr(out["adv"]),
+        _ptr(out["adv_dec"]), _ptr(loss), _ptr(ws), ws.numel(), _stream(stream)))
+    if loss is not None:
+        out["loss"] = loss
+    return out
 
 
 def arbitrate(draft, argmax, stats, w1, b1, w2, b2: float, lam: float, mode: int, p_out, accept,

@@ -11,7 +11,7 @@
 
 namespace cospec {
 
-enum : int { ERR_PAGE = 1, ERR_CTX = 2, ERR_TOKEN = 4, ERR_TIMEOUT = 8 };
+enum : int { ERR_PAGE = 1, ERR_CTX = 2, ERR_TOKEN = 4, ERR_TIMEOUT = 8, ERR_OFFSETS = 16 };
 
 CS_DEV void set_err(int* err, int bit) { atomicOr(err, bit); }
 

@@ -34,7 +34,7 @@ import torch
 
 # tensor ids used in the seed formula config.index * 1000 + id
 _TID = dict(ctx=1, pages=2, q=3, k_blk=4, v_blk=5, k_pages=6, v_pages=7,
-            hidden=8, w=9, mlp=10, drafts=11, sample=12)
+            hidden=8, w=9, mlp=10, drafts=11, sample=12, rl=13)
 
 NUM_FEATURES = 8
 
@@ -283,3 +283,23 @@ def draft_for_rows(draft: np.ndarray) -> np.ndarray:
     out = np.full((B, K + 1), -1, dtype=np.int32)
     out[:, :K] = draft
     return out.reshape(-1)
+
+
+def rl_batch(seed: int, groups: int, rollouts: int, rounds: int, k: int,
+             mismatch_rate: float = 0.3, keep_rate: float = 0.6, correct_rate: float = 0.5):
+    """Synthetic rollout records for the RL stage: ``groups`` prompts with
+    ``rollouts`` rollouts of 1..``rounds`` rounds each; per position a
+    mismatch with probability ``mismatch_rate``, the draft kept at a mismatch
+    with probability ``keep_rate``, log-probabilities -Exp(1.5), a correct
+    rollout with probability ``correct_rate``.  NumPy arrays: group_off,
+    correct, round_off, match, accept, ell."""
+    rng = np.random.default_rng(seed)
+    nr = rng.integers(1, rounds + 1, size=groups * rollouts)
+    round_off = np.concatenate([[0], np.cumsum(nr)]).astype(np.int32)
+    R = int(round_off[-1])
+    match = (rng.random((R, k)) >= mismatch_rate).astype(np.uint8)
+    accept = np.where(match == 1, 1, rng.random((R, k)) < keep_rate).astype(np.uint8)
+    ell = (-rng.exponential(1.5, (R, k))).astype(np.float32)
+    correct = (rng.random(groups * rollouts) < correct_rate).astype(np.uint8)
+    group_off = (np.arange(groups + 1) * rollouts).astype(np.int32)
+    return group_off, correct, round_off, match, accept, ell
