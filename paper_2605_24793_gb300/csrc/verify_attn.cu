@@ -172,7 +172,10 @@ CS_DEV void attend(uint32_t sk, uint32_t sv, uint32_t group_bytes, uint32_t half
   }
 }
 
-template <int D, int MT, int WK>
+// GEN: blocks of more than 32 rows or a full block mask (the arbitrator's
+// region) take a general block path; the verify block (causal, <= 32 rows)
+// keeps a specialised one.
+template <int D, int MT, int WK, bool GEN>
 __global__ void __launch_bounds__(MT* WK * 32 + 32)
     verify_attn_kernel(const __grid_constant__ CUtensorMap map_kp,
                        const __grid_constant__ CUtensorMap map_vp,
@@ -380,13 +383,23 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
       }
       named_bar_sync(1, NTC);
       if (wk == 0) {
-        // causal: block key j is seen by the rows of block rows >= j; full: by every row
-        const int b0 = p.block_full ? p.R - 1 : j0, b1 = p.block_full ? p.R - 1 : j1;
         const uint32_t sk = smem_u32(blk_k), sv = smem_u32(blk_v);
-        // 16 block keys at a time (one code path for any block length)
-        for (int g0 = 0; g0 < KBR; g0 += 16)
-          attend<D, 16>(sk, sv, PAGE * ROWB, KBR * ROWB, g0, g0, true, b0, b1, p.scale_log2, qf, o,
-                        m0, m1, l0, l1, lane);
+        if constexpr (!GEN) {
+          // causal: block key j is seen by the rows of block rows >= j
+          if (KBR == 16)
+            attend<D, 16>(sk, sv, PAGE * ROWB, 16 * ROWB, 0, 0, true, j0, j1, p.scale_log2, qf, o,
+                          m0, m1, l0, l1, lane);
+          else
+            attend<D, 32>(sk, sv, PAGE * ROWB, 32 * ROWB, 0, 0, true, j0, j1, p.scale_log2, qf, o,
+                          m0, m1, l0, l1, lane);
+        } else {
+          // any block length up to 64, causal or full (every block row seen
+          // by every row): 16 keys at a time
+          const int b0 = p.block_full ? p.R - 1 : j0, b1 = p.block_full ? p.R - 1 : j1;
+          for (int g0 = 0; g0 < KBR; g0 += 16)
+            attend<D, 16>(sk, sv, PAGE * ROWB, KBR * ROWB, g0, g0, true, b0, b1, p.scale_log2, qf, o,
+                          m0, m1, l0, l1, lane);
+        }
       }
     }
     // After a timed-out wait a copy may still be in flight: wait (bounded)
@@ -538,7 +551,7 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
 }
 
 
-template <int D, int MT, int WK>
+template <int D, int MT, int WK, bool GEN>
 cudaError_t launch_t(const CUtensorMap* maps, const AttnParams& p, int S, int B, int Hkv,
                      cudaStream_t stream) {
   using LY = Layout<D, MT, WK>;
@@ -549,7 +562,7 @@ cudaError_t launch_t(const CUtensorMap* maps, const AttnParams& p, int S, int B,
   static bool cluster_ok[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
-  auto kern = verify_attn_kernel<D, MT, WK>;
+  auto kern = verify_attn_kernel<D, MT, WK, GEN>;
   if (dev < 64 && configured[dev] < smem) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -580,7 +593,8 @@ cudaError_t launch_t(const CUtensorMap* maps, const AttnParams& p, int S, int B,
 template <int D, int MT, int WK>
 int max_cluster_t(int S, int Hkv, int B, int kbr) {
   using LY = Layout<D, MT, WK>;
-  auto kern = verify_attn_kernel<D, MT, WK>;
+  // both block paths have the same shared-memory layout for a block size
+  auto kern = kbr > 32 ? verify_attn_kernel<D, MT, WK, true> : verify_attn_kernel<D, MT, WK, false>;
   // the occupancy query needs the limit at least at the queried size; it
   // never lowers a limit a launch has raised
   int cur = 0;
@@ -722,7 +736,9 @@ cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& pl, int* err,
   p.err = err;
 #define X(DD, MM, WW)                                      \
   if (a.D == DD && pl.mt == MM && pl.wk == WW)             \
-    return launch_t<DD, MM, WW>(maps, p, pl.cluster, a.B, a.Hkv, stream);
+    return (a.R > 32 || a.block_full)                                                       \
+               ? launch_t<DD, MM, WW, true>(maps, p, pl.cluster, a.B, a.Hkv, stream)           \
+               : launch_t<DD, MM, WW, false>(maps, p, pl.cluster, a.B, a.Hkv, stream);
   COSPEC_ATTN_VARIANTS(X)
 #undef X
   return cudaErrorInvalidValue;
