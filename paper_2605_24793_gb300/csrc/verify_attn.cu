@@ -253,7 +253,9 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
       tma_prefetch_desc(&map_kp);
       tma_prefetch_desc(&map_vp);
     }
-    const uint64_t pol = l2_policy_evict_first();
+    // KV is read once per row group: with several groups per (sequence, head)
+    // (running side by side) keep it in L2 for the siblings
+    const uint64_t pol = p.RG > 1 ? l2_policy_evict_normal() : l2_policy_evict_first();
     bool waited = !p.kv_stable;
     if (do_blk && p.R > 0) {
       // the block K/V is written by the previous kernel: wait first

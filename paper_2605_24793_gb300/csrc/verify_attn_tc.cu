@@ -278,7 +278,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       tma_prefetch_desc(&map_vp);
       tma_prefetch_desc(&map_q);
     }
-    const uint64_t pol = l2_policy_evict_first();
+    // KV is read once per row group: with several groups per (sequence, head)
+    // (running side by side) keep it in L2 for the siblings
+    const uint64_t pol = p.RG > 1 ? l2_policy_evict_normal() : l2_policy_evict_first();
     const int* ptab = p.page_table + (size_t)b * p.max_pages + (size_t)t_begin * TPPT;
     const int my_pages = min(n * TPPT, npages - t_begin * TPPT);
     int pid = 0;
