@@ -25,20 +25,6 @@ CS_DEV uint64_t global_timer_ns() {
   return t;
 }
 
-// ---------------------------------------------------------------- cp.async
-// 16-byte global->shared copy; when !valid nothing is read and the 16 bytes
-// are zero-filled.
-CS_DEV void cp_async16(uint32_t dst, const void* src, bool valid) {
-  int n = valid ? 16 : 0;
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(n)
-               : "memory");
-}
-CS_DEV void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
-template <int N>
-CS_DEV void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
-}
-
 // ---------------------------------------------------------------- ldmatrix / mma.sync
 CS_DEV void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
@@ -179,12 +165,7 @@ CS_DEV uint32_t cluster_nctarank() {
   asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
   return r;
 }
-// Full cluster barrier (every thread of every CTA of the cluster arrives).
-CS_DEV void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n"
-               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-// The two halves of cluster_sync, for work in between (every thread of the
+// Cluster barrier in two halves, for work in between (every thread of the
 // CTA executes both, arrive first).
 CS_DEV void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
 CS_DEV void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
@@ -204,24 +185,6 @@ CS_DEV void bulk_copy_s2s(uint32_t dst_cluster, uint32_t src_cta, uint32_t bytes
           dst_cluster),
       "r"(src_cta), "r"(bytes), "r"(bar_cluster)
       : "memory");
-}
-CS_DEV void dsmem_st_f4(uint32_t addr, float4 v) {
-  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(v.x), "f"(v.y),
-               "f"(v.z), "f"(v.w)
-               : "memory");
-}
-CS_DEV float2 dsmem_ld_f2(uint32_t addr) {
-  float2 v;
-  asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr) : "memory");
-  return v;
-}
-CS_DEV float4 dsmem_ld_f4(uint32_t addr) {
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(addr)
-               : "memory");
-  return v;
 }
 
 // ---------------------------------------------------------------- tcgen05
