@@ -428,71 +428,69 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
   }
 
   // CTA partial: rows of every warp, key groups merged (stage ring reused).
-  // A partial row holds O[0..D) then (m, l) at D, D+1 (fp32, padded to PD).
   float* part = reinterpret_cast<float*>(smem + LY::PART);
-  if constexpr (WK == 1) {
-    if (warp < NWARPS) {
-#pragma unroll
-      for (int nd = 0; nd < D / 8; ++nd) {
-        const int col = nd * 8 + 2 * c4;
-        *reinterpret_cast<float2*>(part + r0 * PD + col) = make_float2(o[nd][0], o[nd][1]);
-        *reinterpret_cast<float2*>(part + r1 * PD + col) = make_float2(o[nd][2], o[nd][3]);
-      }
-      if (c4 == 0) {
-        *reinterpret_cast<float2*>(part + r0 * PD + D) = make_float2(m0, l0);
-        *reinterpret_cast<float2*>(part + r1 * PD + D) = make_float2(m1, l1);
-      }
-    }
-  } else {
+  if constexpr (WK > 1) {
+    // Key groups of a row tile merge pairwise in registers: every lane of a
+    // partner warp holds the same (row, column) elements, so one writes its
+    // (O, m, l) and the other folds them in (a tree over the WK groups).
     float* red = reinterpret_cast<float*>(smem);                          // [NWARPS][16][PD]
-    if (warp < NWARPS) {
-      float* wo = red + warp * 16 * PD;
 #pragma unroll
-      for (int nd = 0; nd < D / 8; ++nd) {
-        const int col = nd * 8 + 2 * c4;
-        *reinterpret_cast<float2*>(wo + g_row * PD + col) = make_float2(o[nd][0], o[nd][1]);
-        *reinterpret_cast<float2*>(wo + (g_row + 8) * PD + col) = make_float2(o[nd][2], o[nd][3]);
+    for (int step = 1; step < WK; step <<= 1) {
+      const bool writer = warp < NWARPS && (wk % (2 * step)) == step;
+      const bool reader = warp < NWARPS && (wk % (2 * step)) == 0;
+      if (writer) {
+        float* wo = red + warp * 16 * PD;
+#pragma unroll
+        for (int nd = 0; nd < D / 8; ++nd) {
+          const int col = nd * 8 + 2 * c4;
+          *reinterpret_cast<float2*>(wo + g_row * PD + col) = make_float2(o[nd][0], o[nd][1]);
+          *reinterpret_cast<float2*>(wo + (g_row + 8) * PD + col) = make_float2(o[nd][2], o[nd][3]);
+        }
+        if (c4 == 0) {
+          *reinterpret_cast<float2*>(wo + g_row * PD + D) = make_float2(m0, l0);
+          *reinterpret_cast<float2*>(wo + (g_row + 8) * PD + D) = make_float2(m1, l1);
+        }
       }
-      if (c4 == 0) {
-        *reinterpret_cast<float2*>(wo + g_row * PD + D) = make_float2(m0, l0);
-        *reinterpret_cast<float2*>(wo + (g_row + 8) * PD + D) = make_float2(m1, l1);
+      __syncthreads();
+      if (reader) {
+        const float* po = red + (warp + step) * 16 * PD;
+        const float2 ml0 = *reinterpret_cast<const float2*>(po + g_row * PD + D);
+        const float2 ml1 = *reinterpret_cast<const float2*>(po + (g_row + 8) * PD + D);
+        const float M0 = fmaxf(m0, ml0.x), M1 = fmaxf(m1, ml1.x);
+        const float a0 = (M0 == -INFINITY) ? 0.f : exp2_approx(m0 - M0);
+        const float b0 = (M0 == -INFINITY) ? 0.f : exp2_approx(ml0.x - M0);
+        const float a1 = (M1 == -INFINITY) ? 0.f : exp2_approx(m1 - M1);
+        const float b1 = (M1 == -INFINITY) ? 0.f : exp2_approx(ml1.x - M1);
+#pragma unroll
+        for (int nd = 0; nd < D / 8; ++nd) {
+          const int col = nd * 8 + 2 * c4;
+          const float2 v0 = *reinterpret_cast<const float2*>(po + g_row * PD + col);
+          const float2 v1 = *reinterpret_cast<const float2*>(po + (g_row + 8) * PD + col);
+          o[nd][0] = o[nd][0] * a0 + v0.x * b0;
+          o[nd][1] = o[nd][1] * a0 + v0.y * b0;
+          o[nd][2] = o[nd][2] * a1 + v1.x * b1;
+          o[nd][3] = o[nd][3] * a1 + v1.y * b1;
+        }
+        l0 = l0 * a0 + ml0.y * b0;
+        l1 = l1 * a1 + ml1.y * b1;
+        m0 = M0;
+        m1 = M1;
       }
+      if (2 * step < WK) __syncthreads();   // the next level reuses the buffer
     }
-    __syncthreads();
-    // Per row: the common maximum, each key group's weight and the total sum,
-    // computed once (kept in the partial row's (m, l) slots) ...
-    for (int r = tid; r < NRP; r += NTT) {
-      const int rt = r / 16, ri = r % 16;
-      float M = -INFINITY;
+  }
+  // The first key group of every row tile (all warps when WK == 1) writes
+  // the CTA's partial rows: O[0..D) then (m, l) at D, D+1 (fp32, padded to PD).
+  if (warp < NWARPS && wk == 0) {
 #pragma unroll
-      for (int w = 0; w < WK; ++w) M = fmaxf(M, red[((rt * WK + w) * 16 + ri) * PD + D]);
-      float L = 0.f;
-#pragma unroll
-      for (int w = 0; w < WK; ++w) {
-        float* wr_ = red + ((rt * WK + w) * 16 + ri) * PD;
-        const float sc = (M == -INFINITY) ? 0.f : exp2_approx(wr_[D] - M);
-        L += wr_[D + 1] * sc;
-        wr_[D + 2] = sc;
-      }
-      *reinterpret_cast<float2*>(part + r * PD + D) = make_float2(M, L);
+    for (int nd = 0; nd < D / 8; ++nd) {
+      const int col = nd * 8 + 2 * c4;
+      *reinterpret_cast<float2*>(part + r0 * PD + col) = make_float2(o[nd][0], o[nd][1]);
+      *reinterpret_cast<float2*>(part + r1 * PD + col) = make_float2(o[nd][2], o[nd][3]);
     }
-    __syncthreads();
-    // ... then every output chunk is a weighted sum of the key groups' chunks.
-    for (int e = tid; e < NRP * (D / 4); e += NTT) {
-      const int r = e / (D / 4), c = (e % (D / 4)) * 4;
-      const int rt = r / 16, ri = r % 16;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-      for (int w = 0; w < WK; ++w) {
-        const float* wr_ = red + ((rt * WK + w) * 16 + ri) * PD;
-        const float sc = wr_[D + 2];
-        const float4 v = *reinterpret_cast<const float4*>(wr_ + c);
-        acc.x += v.x * sc;
-        acc.y += v.y * sc;
-        acc.z += v.z * sc;
-        acc.w += v.w * sc;
-      }
-      *reinterpret_cast<float4*>(part + r * PD + c) = acc;
+    if (c4 == 0) {
+      *reinterpret_cast<float2*>(part + r0 * PD + D) = make_float2(m0, l0);
+      *reinterpret_cast<float2*>(part + r1 * PD + D) = make_float2(m1, l1);
     }
   }
   fence_proxy_async_smem();              // the bulk copies below read `part`
