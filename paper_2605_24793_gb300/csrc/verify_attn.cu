@@ -519,32 +519,42 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
     cluster_arrive();
   }
   const int row0 = rank * rpo;
+  // Per owned row: one warp forms the common maximum over the S partials and
+  // each partial's weight exp2(m_s - M) / L (kept in the idle block region);
+  // then every output chunk is a plain weighted sum.
+  float* scl = reinterpret_cast<float*>(blk_k);            // [S][rpo]
+  for (int rr = warp; rr < rpo; rr += NTT / 32) {
+    if (row0 + rr >= NR) break;
+    const float2 ml = (lane < S) ? *reinterpret_cast<const float2*>(src + (lane * rpo + rr) * PD + D)
+                                 : make_float2(-INFINITY, 0.f);
+    float M = ml.x;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    const float sc = (M == -INFINITY || ml.x == -INFINITY) ? 0.f : exp2_approx(ml.x - M);
+    float L = ml.y * sc;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) L += __shfl_xor_sync(0xffffffffu, L, off);
+    if (lane < S) scl[lane * rpo + rr] = (L > 0.f) ? sc / L : 0.f;
+  }
+  __syncthreads();
   for (int e = tid; e < rpo * (D / 4); e += NTT) {
     const int rr = e / (D / 4), c = (e % (D / 4)) * 4;
     const int r = row0 + rr;
     if (r >= NR) break;
-    float M = -INFINITY;
-    for (int s2 = 0; s2 < S; ++s2) M = fmaxf(M, src[(s2 * rpo + rr) * PD + D]);
-    float L = 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (M != -INFINITY) {
-      for (int s2 = 0; s2 < S; ++s2) {
-        const float* pr = src + (s2 * rpo + rr) * PD;
-        const float sc = exp2_approx(pr[D] - M);
-        L += pr[D + 1] * sc;
-        const float4 v = *reinterpret_cast<const float4*>(pr + c);
-        acc.x += v.x * sc;
-        acc.y += v.y * sc;
-        acc.z += v.z * sc;
-        acc.w += v.w * sc;
-      }
+    for (int s2 = 0; s2 < S; ++s2) {
+      const float w = scl[s2 * rpo + rr];
+      const float4 v = *reinterpret_cast<const float4*>(src + (s2 * rpo + rr) * PD + c);
+      acc.x += v.x * w;
+      acc.y += v.y * w;
+      acc.z += v.z * w;
+      acc.w += v.w * w;
     }
-    const float inv = (L > 0.f) ? 1.f / L : 0.f;
     const int j = (row_g0 + r) / p.G, g = (row_g0 + r) % p.G;
     __nv_bfloat16* dst = p.out + (((size_t)b * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D + c;
     uint2 pk;
-    pk.x = pack_bf16(acc.x * inv, acc.y * inv);
-    pk.y = pack_bf16(acc.z * inv, acc.w * inv);
+    pk.x = pack_bf16(acc.x, acc.y);
+    pk.y = pack_bf16(acc.z, acc.w);
     *reinterpret_cast<uint2*>(dst) = pk;
   }
   if (S > 1) cluster_wait();             // every copy out of this CTA has landed
