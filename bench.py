@@ -283,6 +283,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--layers", type=int, default=None, help="override the layer count")
+    ap.add_argument("--k", type=int, default=None,
+                    help="override the draft length K (block rows K+1), e.g. 25 as in the paper")
     ap.add_argument("--temperature", type=float, default=None,
                     help="stochastic decoding: sample the target candidates at this temperature")
     args = ap.parse_args()
@@ -309,10 +311,14 @@ def main():
     cfg = W.CONFIGS[args.config]
     if args.layers:
         cfg = cfg.replace(layers=args.layers)
+    if args.k is not None:
+        cfg = cfg.replace(k=args.k)
     inp = W.make_round_inputs(cfg, device="cuda")
     draft = gpu_drafts(cfg, inp)
     rnd = VerifyRound(inp, draft, cfg.lam, temperature=args.temperature,
                       seed=W.sample_seed(cfg))
+    attn_kernel, attn_splits = C.verify_attn_plan(inp["q"][0], inp["k_pages"][0], inp["page_table"],
+                                                  rnd.max_ctx)
     lm_name = "lmhead_argmax_features" if args.temperature is None else "lmhead_sample_features"
     stream = torch.cuda.Stream()
     torch.cuda.synchronize()
@@ -420,6 +426,8 @@ def main():
     lm_t_tc = lmhead_flops(cfg) / (tflops_peak * 1e12)
     kern = {
         "verify_attn": {"ms_per_launch": attn_launch_ms, "launches_per_step": cfg.layers,
+                        "kernel": "tcgen05" if attn_kernel == C.ATTN_TCGEN05 else "mma.sync",
+                        "splits": attn_splits,
                         "bytes_per_launch": a_bytes,
                         "gbs": a_bytes / (attn_launch_ms * 1e-3) / 1e9,
                         "frac_hbm": a_bytes / (attn_launch_ms * 1e-3) / 1e9 / hbm,

@@ -138,28 +138,33 @@ static int check_attn_dims(const cospec_attn_dims* d) {
   return COSPEC_OK;
 }
 
-// Largest schedulable cluster not above `S` for this variant (cached per device).
-static int schedulable_cluster(int D, const AttnPlan& pl, int Hkv, int B, int R) {
-  // [dev][D==128][variant][block keys / 16 - 1][log2 S] : 0 unknown, 1 ok, -1 no
-  static int cache[64][2][6][4][5];
+// Clusters of S CTAs of a plan's attention variant resident at once (the
+// occupancy query, cached per device; it depends on the variant and its shared
+// memory, not on the grid).
+static long long resident_clusters(int D, const AttnPlan& pl, int S, int Hkv, int B, int R) {
+  // [dev][D==128][variant][block keys / 16 - 1][log2 S]: count + 1 (0: not yet queried)
+  static int cache[MAX_DEV][2][6][4][5];
   const int kbr = (R + 15) & ~15;
   int dev = 0;
   cudaGetDevice(&dev);
   const int di = D == 128 ? 1 : 0;
   const int mi = pl.kind == 1 ? (pl.nt == 32 ? 4 : 5)
                               : (pl.mt == 1 ? 0 : pl.mt == 2 ? 1 : pl.mt == 4 ? 2 : 3);
-  int S = pl.cluster;
-  while (S > 1) {
-    int ls = 0;
-    while ((1 << ls) < S) ++ls;
-    int& c = cache[dev < 64 ? dev : 63][di][mi][kbr / 16 - 1][ls];
-    if (c == 0)
-      c = (pl.kind == 1 ? attn_tc_max_active_clusters(D, pl.nt, S, Hkv, B, pl.rg)
-                        : attn_max_active_clusters(D, pl.mt, pl.wk, S, Hkv, B, kbr)) > 0 ? 1 : -1;
-    if (c > 0) break;
-    S >>= 1;
-  }
-  return S;
+  int ls = 0;
+  while ((1 << ls) < S) ++ls;
+  int& c = cache[dev < MAX_DEV ? dev : MAX_DEV - 1][di][mi][kbr / 16 - 1][ls];
+  if (c == 0)
+    c = 1 + (pl.kind == 1 ? attn_tc_max_active_clusters(D, pl.nt, S, Hkv, B, pl.rg)
+                          : attn_max_active_clusters(D, pl.mt, pl.wk, S, Hkv, B, kbr));
+  return c - 1;
+}
+
+static AttnPlan attn_plan(const cospec_attn_dims* d, int max_ctx, int sms) {
+  return plan_verify_attn(d->batch, d->rows, d->num_q_heads, d->num_kv_heads, d->head_dim,
+                          max_ctx, sms, [d](const AttnPlan& pl, int S) {
+                            return resident_clusters(d->head_dim, pl, S, d->num_kv_heads,
+                                                     d->batch > 0 ? d->batch : 1, d->rows);
+                          });
 }
 
 COSPEC_API int cospec_verify_attn_plan(const cospec_attn_dims* d, int max_ctx, int* kernel,
@@ -170,9 +175,7 @@ COSPEC_API int cospec_verify_attn_plan(const cospec_attn_dims* d, int max_ctx, i
   CS_CHECK_ARG(max_ctx >= 0 && max_ctx <= d->max_pages_per_seq * d->page_size);
   const int sms = device_num_sms();
   if (sms <= 0) return COSPEC_ERR_CUDA;
-  AttnPlan pl = plan_verify_attn(d->batch, d->rows, d->num_q_heads, d->num_kv_heads,
-                                 d->head_dim, max_ctx, sms);
-  pl.cluster = schedulable_cluster(d->head_dim, pl, d->num_kv_heads, d->batch, d->rows);
+  const AttnPlan pl = attn_plan(d, max_ctx, sms);
   *kernel = pl.kind;
   *splits = pl.cluster;
   return COSPEC_OK;
@@ -192,9 +195,7 @@ COSPEC_API int cospec_verify_attn(const cospec_attn_dims* d, int max_ctx, const 
                aligned16(v_pages) && aligned16(out));
   const int sms = device_num_sms();
   if (sms <= 0) return COSPEC_ERR_CUDA;
-  AttnPlan pl = plan_verify_attn(d->batch, d->rows, d->num_q_heads, d->num_kv_heads,
-                                 d->head_dim, max_ctx, sms);
-  pl.cluster = schedulable_cluster(d->head_dim, pl, d->num_kv_heads, d->batch, d->rows);
+  const AttnPlan pl = attn_plan(d, max_ctx, sms);
   int* err = device_error_word();
   if (!err) return COSPEC_ERR_CUDA;
   AttnArgs a{};

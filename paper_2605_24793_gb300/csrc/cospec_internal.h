@@ -4,6 +4,7 @@
 
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
+#include <functional>
 #include <stddef.h>
 #include <stdint.h>
 
@@ -59,10 +60,15 @@ struct AttnPlan {
   int nt, jb, jbq, rg;    // tcgen05: row capacity (32 / 64), block rows per row group,
                           // block rows of the query box, row groups
   int cluster;            // CTAs per (sequence, KV head, row group): the KV split
-  int tiles_per_split, max_splits;
-  size_t total_bytes;     // workspace (none)
+  long long units;        // (sequence, KV head, row group) units, one cluster each
+  int one_wave;           // small batch: take the largest split whose clusters are
+                          // all resident at once (latency-bound)
 };
-AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int num_sms);
+// Clusters of `S` CTAs of the plan's kernel variant resident at once on the
+// device (0: not schedulable).
+using ResidentFn = std::function<long long(const AttnPlan&, int S)>;
+AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int num_sms,
+                          const ResidentFn& resident);
 int attn_max_active_clusters(int D, int mt, int wk, int S, int Hkv, int B, int kbr);
 cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& plan, int* err,
                                cudaStream_t stream);

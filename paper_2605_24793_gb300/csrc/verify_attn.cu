@@ -643,7 +643,8 @@ int variant_mt(int NR) {   // NR <= 64
 
 }  // namespace
 
-AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int num_sms) {
+AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int num_sms,
+                          const ResidentFn& resident) {
   AttnPlan pl{};
   const int NRT = (Hq / Hkv) * R;
   const int RG = (NRT + 63) / 64;                  // row groups of at most 64 rows
@@ -651,21 +652,6 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
   pl.mt = variant_mt(NR);
   pl.wk = (pl.mt >= 4) ? 1 : 4 / pl.mt;
   pl.nrp = pl.mt * 16;
-  // Split each (sequence, head) over a cluster of S CTAs: about one wave at
-  // two CTAs per SM, no CTA with more than 256 cache tiles (long contexts),
-  // at least 4 tiles per CTA, at most 16 CTAs per cluster.
-  const int tiles = (max_ctx + KT - 1) / KT;
-  const long long units = (long long)B * Hkv * RG;
-  const long long want_wave = (2LL * num_sms + units - 1) / (units > 0 ? units : 1);
-  const long long want_len = (tiles + 255) / 256;
-  const long long want = want_wave > want_len ? want_wave : want_len;
-  int S = 1;
-  while (S < 16 && S < want && (S * 2) * 4 <= tiles) S *= 2;
-  pl.kind = 0;
-  pl.cluster = S;
-  pl.tiles_per_split = (tiles + S - 1) / S;
-  pl.max_splits = S;
-  pl.total_bytes = 0;
   const int G = Hq / Hkv;
   const int jb = G <= 64 ? 64 / G : 1;
   const int jbq = R < jb ? R : jb;
@@ -674,6 +660,7 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
   // rate there, and the tcgen05 kernel (one CTA per SM, deep ring) takes
   // over.  Small batches stay latency-bound and keep the mma.sync kernel.
   const long long units_g = (long long)B * Hkv * ((R + jb - 1) / jb);
+  int S = 1;
   if (tc_attn_supported(D, G) && G * jbq > 32 && units_g >= num_sms) {
     // tcgen05 kernel: row groups of whole block rows, at most 64 query rows
     pl.kind = 1;
@@ -685,16 +672,39 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
     // least two tiles per CTA, no CTA with more than 64 tiles (long
     // sequences split, so that uneven contexts balance over the waves).
     const int tiles_tc = (max_ctx + 127) / 128;
-    const long long units_tc = (long long)B * Hkv * pl.rg;
-    const long long wave_tc = ((long long)num_sms + units_tc - 1) / (units_tc > 0 ? units_tc : 1);
+    pl.units = (long long)B * Hkv * pl.rg;
+    const long long wave_tc = ((long long)num_sms + pl.units - 1) / (pl.units > 0 ? pl.units : 1);
     const long long len_tc = (tiles_tc + 63) / 64;
     const long long want_tc = wave_tc > len_tc ? wave_tc : len_tc;
-    int St = 1;
-    while (St < 16 && St < want_tc && (St * 2) * 2 <= tiles_tc) St *= 2;
-    pl.cluster = St;
-    pl.tiles_per_split = (tiles_tc + St - 1) / St;
-    pl.max_splits = St;
+    while (S < 16 && S < want_tc && (S * 2) * 2 <= tiles_tc) S *= 2;
+  } else {
+    // Split each (sequence, head, row group) over a cluster of S CTAs: about
+    // one wave of CTAs (as many as are resident at once), no CTA with more
+    // than 256 cache tiles (long contexts), at least 4 tiles per CTA, at
+    // most 16 CTAs per cluster.
+    pl.kind = 0;
+    const int tiles = (max_ctx + KT - 1) / KT;
+    pl.units = (long long)B * Hkv * RG;
+    long long slots = resident(pl, 1);
+    if (slots < 1) slots = num_sms;
+    const long long want_wave = (slots + pl.units - 1) / (pl.units > 0 ? pl.units : 1);
+    const long long want_len = (tiles + 255) / 256;
+    const long long want = want_wave > want_len ? want_wave : want_len;
+    while (S < 16 && S < want && (S * 2) * 4 <= tiles) S *= 2;
+    // A batch of a few units (at most a quarter of the slots) is bound by the
+    // latency of one CTA's tile loop and the cluster merge, and a second wave
+    // of clusters (the GPU places whole clusters inside one GPC) doubles it:
+    // take the largest split whose clusters are all resident at once.
+    pl.one_wave = (pl.units * 4 <= slots && want_len <= 1) ? 1 : 0;
   }
+  // the largest cluster not above S that can be scheduled at all (and, for a
+  // one-wave launch, with every cluster resident)
+  while (S > 1) {
+    const long long n = resident(pl, S);
+    if (n > 0 && (!pl.one_wave || n >= pl.units)) break;
+    S >>= 1;
+  }
+  pl.cluster = S;
   return pl;
 }
 
