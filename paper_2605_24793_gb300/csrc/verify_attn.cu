@@ -64,11 +64,15 @@ struct Layout {
   static constexpr int RECV = PART_END;
   static constexpr int RECV_END = RECV + (NRP + 15) * ROWP;
   static_assert(RECV_END <= NSTAGE * STAGE, "partials must fit in the stage ring");
-  static constexpr int BAR = NSTAGE * STAGE;       // full[NSTAGE], empty[NSTAGE], block
-  static constexpr int BLK = BAR + (2 * NSTAGE + 2) * 8 + 1024;   // 1024-aligned block K/V
+  static constexpr int BLK = NSTAGE * STAGE;       // block K/V (1024-aligned)
   // the block region holds 2*H halves of KBR rows (KBR = 16, 32, 48 or 64, runtime)
   static constexpr int blk_half(int kbr) { return kbr * ROWB; }
-  static constexpr int total(int kbr) { return BLK / 1024 * 1024 + 2 * H * kbr * ROWB; }
+  static constexpr int total(int kbr) { return BLK + 2 * H * kbr * ROWB; }
+  // The launch adds 1024 bytes to align the base; the 2*NSTAGE+2 barriers
+  // (full[NSTAGE], empty[NSTAGE], block, received partials) take 64 bytes of
+  // that slack, before the aligned base or after the end, whichever side has
+  // room, so that two CTAs of 32 block rows still share one SM.
+  static constexpr int NBAR_BYTES = (2 * NSTAGE + 2) * 8;
 };
 
 // Shared-memory byte offset of 16-byte chunk `ch` (of D/8) of key row `key`
@@ -172,11 +176,18 @@ CS_DEV void attend(uint32_t sk, uint32_t sv, uint32_t group_bytes, uint32_t half
   }
 }
 
-// GEN: blocks of more than 32 rows or a full block mask (the arbitrator's
-// region) take a general block path; the verify block (causal, <= 32 rows)
-// keeps a specialised one.
-template <int D, int MT, int WK, bool GEN>
-__global__ void __launch_bounds__(MT* WK * 32 + 32)
+// GEN 0: the verify block (causal, <= 32 rows), a specialised block path.
+// GEN 1 / 2: blocks of more than 32 rows or a full block mask (the
+// arbitrator's region) take a general block path; 2 marks more than 32 block
+// keys in the 64-row variant.
+// The 64-row variant with at most 32 block keys declares room for two CTAs of
+// six warps per SM, which holds it at 168 registers: two of its five-warp
+// CTAs then fit the register file of each SM sub-partition (three warps of
+// 168).  With more block keys the shared memory allows one CTA per SM, and
+// it keeps its registers (no spills).
+template <int D, int MT, int WK, int GEN>
+__global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 32,
+                                  MT >= 4 && GEN < 2 ? 2 : 0)
     verify_attn_kernel(const __grid_constant__ CUtensorMap map_kp,
                        const __grid_constant__ CUtensorMap map_vp,
                        const __grid_constant__ CUtensorMap map_kb,
@@ -191,14 +202,15 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
   constexpr int PD = LY::PD;
   static_assert(KW % 16 == 0, "keys per warp must be a multiple of 16");
 
-  extern __shared__ uint8_t smem_raw[];
+  extern __shared__ __align__(16) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + LY::BAR);
+  uint64_t* full = reinterpret_cast<uint64_t*>(
+      smem - smem_raw >= LY::NBAR_BYTES ? smem_raw : smem + LY::total((p.R + 15) & ~15));
   uint64_t* empty = full + NSTAGE;
   uint64_t* blk_full = empty + NSTAGE;
   uint64_t* recv_bar = blk_full + 1;     // partials received from the cluster
-  uint8_t* blk_k = smem + LY::BLK / 1024 * 1024;          // block keys: 2*H halves of KBR rows
+  uint8_t* blk_k = smem + LY::BLK;       // block keys: 2*H halves of KBR rows
 
   const int S = (int)cluster_nctarank();
   const int rank = (int)cluster_ctarank();
@@ -386,7 +398,7 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
       named_bar_sync(1, NTC);
       if (wk == 0) {
         const uint32_t sk = smem_u32(blk_k), sv = smem_u32(blk_v);
-        if constexpr (!GEN) {
+        if constexpr (GEN == 0) {
           // causal: block key j is seen by the rows of block rows >= j
           if (KBR == 16)
             attend<D, 16>(sk, sv, PAGE * ROWB, 16 * ROWB, 0, 0, true, j0, j1, p.scale_log2, qf, o,
@@ -561,7 +573,7 @@ __global__ void __launch_bounds__(MT* WK * 32 + 32)
 }
 
 
-template <int D, int MT, int WK, bool GEN>
+template <int D, int MT, int WK, int GEN>
 cudaError_t launch_t(const CUtensorMap* maps, const AttnParams& p, int S, int B, int Hkv,
                      cudaStream_t stream) {
   using LY = Layout<D, MT, WK>;
@@ -603,8 +615,10 @@ cudaError_t launch_t(const CUtensorMap* maps, const AttnParams& p, int S, int B,
 template <int D, int MT, int WK>
 int max_cluster_t(int S, int Hkv, int B, int kbr) {
   using LY = Layout<D, MT, WK>;
-  // both block paths have the same shared-memory layout for a block size
-  auto kern = kbr > 32 ? verify_attn_kernel<D, MT, WK, true> : verify_attn_kernel<D, MT, WK, false>;
+  // every block path has the same shared-memory layout for a block size, and
+  // the paths used with a block size the same register budget
+  auto kern = kbr > 32 ? verify_attn_kernel<D, MT, WK, (MT >= 4 ? 2 : 1)>
+                       : verify_attn_kernel<D, MT, WK, 0>;
   // the occupancy query needs the limit at least at the queried size; it
   // never lowers a limit a launch has raised
   int cur = 0;
@@ -754,11 +768,14 @@ cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& pl, int* err,
   p.kv_stable = a.kv_stable;
   p.block_full = a.block_full;
   p.err = err;
-#define X(DD, MM, WW)                                      \
-  if (a.D == DD && pl.mt == MM && pl.wk == WW)             \
-    return (a.R > 32 || a.block_full)                                                       \
-               ? launch_t<DD, MM, WW, true>(maps, p, pl.cluster, a.B, a.Hkv, stream)           \
-               : launch_t<DD, MM, WW, false>(maps, p, pl.cluster, a.B, a.Hkv, stream);
+  const bool general = a.R > 32 || a.block_full;
+  const bool wide = ((a.R + 15) & ~15) > 32;
+#define X(DD, MM, WW)                                                                    \
+  if (a.D == DD && pl.mt == MM && pl.wk == WW)                                           \
+    return !general ? launch_t<DD, MM, WW, 0>(maps, p, pl.cluster, a.B, a.Hkv, stream)    \
+           : (MM >= 4 && wide)                                                           \
+               ? launch_t<DD, MM, WW, (MM >= 4 ? 2 : 1)>(maps, p, pl.cluster, a.B, a.Hkv, stream) \
+               : launch_t<DD, MM, WW, 1>(maps, p, pl.cluster, a.B, a.Hkv, stream);
   COSPEC_ATTN_VARIANTS(X)
 #undef X
   return cudaErrorInvalidValue;
