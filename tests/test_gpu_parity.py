@@ -122,6 +122,35 @@ def test_verify_attention_tcgen05_matches_oracle(case):
     assert torch.equal(out, out2)
 
 
+# Long contexts split the tcgen05 kernel's KV range over a cluster (a CTA
+# takes at most 64 tiles of 128 keys): 2, 4 and 8 splits merged through
+# distributed shared memory, with most sequences far shorter than the split.
+ATTN_TC_SPLIT_CASES = [
+    # B, R, Hq, Hkv, D, contexts, shuffled, expected splits
+    (20, 8, 64, 8, 128, [9000] + _ctx(19, 8), True, 2),
+    (20, 16, 32, 8, 128, [20000, 3000] + _ctx(18, 9), True, 4),
+    (20, 8, 64, 8, 128, [33000, 9000] + _ctx(18, 10), False, 8),
+]
+
+
+@pytest.mark.parametrize("case", ATTN_TC_SPLIT_CASES, ids=lambda c: f"B{c[0]}R{c[1]}S{c[7]}")
+def test_verify_attention_tcgen05_split_matches_oracle(case):
+    B, R, Hq, Hkv, D, ctx, shuffled, splits = case
+    rng = np.random.default_rng(B * 1000 + R * 100 + Hq + D + int(sum(ctx)))
+    t = _paged_case(rng, B, R, Hq, Hkv, D, ctx, shuffled)
+    max_ctx = int(max(ctx))
+    jb = 64 // (Hq // Hkv)
+    if C.num_sms() > B * Hkv * (-(-R // jb)):
+        pytest.skip("more SMs than (sequence, head, row group) units on this device")
+    assert C.verify_attn_plan(t["q"], t["k_pages"], t["page_table"], max_ctx) == (C.ATTN_TCGEN05, splits)
+    out = torch.empty_like(t["q"])
+    C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
+                  t["ctx_len"], out, max_ctx)
+    ref = O.verify_attention(host(t["q"]), host(t["k_blk"]), host(t["v_blk"]), host(t["k_pages"]),
+                             host(t["v_pages"]), t["table_np"], t["ctx_np"], 16)
+    assert_close(host(out), ref, "attention (tcgen05, split)")
+
+
 # The arbitrator's draft/target region (Sec. 3.3): 2K+3 block rows that see
 # the whole block; K = 7 gives 17 rows, K = 25 (the paper's default) 53.
 ATTN_FULL_CASES = [
