@@ -15,10 +15,12 @@
 //                 O^T += V^T P^T (M = D, N = query rows, K = keys; V^T is
 //                               read MN-major straight from the V tile);
 //               S^T is double-buffered in TMEM, O^T accumulates in TMEM;
-//   warps 2-5   softmax: one thread per key (TMEM lane) turns a tile of S^T
+//   warps 2-9   softmax: one thread per key (TMEM lane) turns a tile of S^T
 //               into P^T (bf16, written over the tile's K, which the MMA no
 //               longer needs), rescales O^T when needed and reads it out at
-//               the end.
+//               the end.  Two warps share each TMEM lane quarter and split
+//               the query-row columns, so every SM sub-partition holds two
+//               softmax warps that hide each other's latencies.
 // Keys are the MMA M dimension because a verify block has few query rows
 // (G * (K+1)): spreading keys over threads keeps every softmax lane busy.
 //
@@ -41,7 +43,8 @@ constexpr int TKT = 128;          // keys per cache tile (8 pages) = MMA M
 constexpr int TPPT = TKT / 16;    // pages per tile
 constexpr int TPAGE = 16;         // page size (fixed)
 constexpr int TROWB = 128;        // bytes of one swizzled smem row
-constexpr int TC_THREADS = 192;   // producer warp, MMA warp, 4 softmax warps
+constexpr int TC_THREADS = 320;   // producer warp, MMA warp, 8 softmax warps
+constexpr int TC_SOFT = 256;      // softmax threads
 constexpr float LAZY_LOG2 = 8.f;  // rescale only when a score exceeds m_ref by this (log2)
 constexpr uint64_t TC_WAIT_NS = 2000000000ull;
 
@@ -76,8 +79,8 @@ struct TcLayout {
   // mma_done, recv_bar
   static constexpr int NBAR = 2 * NS + 10;
   static constexpr int HOLDER = MISC + NBAR * 8;            // TMEM base address
-  static constexpr int FLAGS = HOLDER + 16;                 // int [2][4] votes, [2] rescale, abort
-  static constexpr int MREF = FLAGS + 64;                   // float [NT] reference maxima
+  static constexpr int FLAGS = HOLDER + 16;                 // int [2][8] votes, [2] rescale, abort
+  static constexpr int MREF = FLAGS + 128;                  // float [NT] reference maxima
   static constexpr int ALPHA = MREF + NT * 4;               // float [NT]
   static constexpr int RED = ALPHA + NT * 4;                // float [4][NT]
   static constexpr int LSUM = RED + 4 * NT * 4;             // float [NT]
@@ -196,10 +199,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   uint64_t* mma_done = pv_done + 1;
   uint64_t* recv_bar = mma_done + 1;  // partials received from the cluster
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(smem + LY::HOLDER);
-  volatile int* votes = reinterpret_cast<volatile int*>(smem + LY::FLAGS);   // [2][4]
-  volatile int* resc = votes + 8;                                             // [2]
-  volatile int* abort_flag = votes + 10;
-  volatile int* n_issued = votes + 11;     // tiles the producer loaded (abort tail)
+  volatile int* votes = reinterpret_cast<volatile int*>(smem + LY::FLAGS);   // [2][8]
+  volatile int* resc = votes + 16;                                            // [2]
+  volatile int* abort_flag = votes + 18;
+  volatile int* n_issued = votes + 19;     // tiles the producer loaded (abort tail)
   float* m_ref = reinterpret_cast<float*>(smem + LY::MREF);
   float* alpha_s = reinterpret_cast<float*>(smem + LY::ALPHA);
   float* red = reinterpret_cast<float*>(smem + LY::RED);
@@ -230,7 +233,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     mbar_init(pv_done, 1);
     mbar_init(mma_done, 1);
     mbar_init(recv_bar, 1);
-    for (int i = 0; i < 12; ++i) votes[i] = 0;
+    for (int i = 0; i < 20; ++i) votes[i] = 0;
     fence_barrier_init();
   }
   if (warp == 1) {
@@ -374,10 +377,19 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       const uint32_t idesc_pv = idesc_bf16_f32(128, N) | (1u << 15);   // A (V^T) MN-major
       const uint32_t q0 = smem_u32(qs);
       bool ok = mbar_wait(q_full, 0, TC_WAIT_NS);
-      auto pv = [&](int u) -> bool {
-        if (!mbar_wait(&p_full[u & 1], (uint32_t)(u >> 1) & 1u, TC_WAIT_NS) || *abort_flag)
-          return false;
-        tc_fence_after();
+      auto issue_s = [&](int t) {
+        const int st = t % NS;
+        const uint32_t kb = smem_u32(smem + st * LY::STAGE);
+        const uint32_t khalf = (do_blk && t == n) ? (uint32_t)(KBR * TROWB) : (uint32_t)(TKT * TROWB);
+#pragma unroll
+        for (int h = 0; h < H; ++h)
+#pragma unroll
+          for (int ks = 0; ks < 4; ++ks)
+            umma_bf16(tmem_base + (uint32_t)((t & 1) * NT), smem_desc_sw128(kb + h * khalf + ks * 32),
+                      smem_desc_sw128(q0 + h * LY::QH + ks * 32), idesc_qk, (h | ks) != 0 ? 1u : 0u);
+        umma_commit(&s_full[t & 1]);
+      };
+      auto issue_pv = [&](int u) {
         const int st = u % NS;
         const uint32_t kb = smem_u32(smem + st * LY::STAGE);
         const bool blk = do_blk && u == n;
@@ -391,35 +403,35 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     (u > 0 || ks > 0) ? 1u : 0u);
         umma_commit(&empty[st]);
         umma_commit(pv_done);
-        return true;
       };
-      for (int t = 0; t < T && ok; ++t) {
-        const int st = t % NS;
-        if (!mbar_wait(&full[st], (uint32_t)(t / NS) & 1u, TC_WAIT_NS) || *abort_flag) {
-          ok = false;
-          break;
+      // Issue whichever product is ready, so that a P.V product (which frees
+      // a ring stage for the producer) never waits behind the next tile's
+      // load.  S^T of tile ts needs the tile and a free S^T buffer; at most
+      // one tile's S^T runs ahead of the oldest pending P.V, which also keeps
+      // every barrier within one phase of the parity tested here.
+      int ts = 0, tp = 0;
+      uint64_t t_last = global_timer_ns();
+      while (ok && tp < T) {
+        bool did = false;
+        if (tp < ts && mbar_test(&p_full[tp & 1], (uint32_t)(tp >> 1) & 1u)) {
+          tc_fence_after();
+          issue_pv(tp);
+          ++tp;
+          did = true;
         }
-        if (t >= 2 &&
-            (!mbar_wait(&s_empty[t & 1], (uint32_t)((t >> 1) - 1) & 1u, TC_WAIT_NS) || *abort_flag)) {
-          ok = false;
-          break;
+        if (ts < T && ts <= tp + 1 && mbar_test(&full[ts % NS], (uint32_t)(ts / NS) & 1u) &&
+            (ts < 2 || mbar_test(&s_empty[ts & 1], (uint32_t)((ts >> 1) - 1) & 1u))) {
+          tc_fence_after();
+          issue_s(ts);
+          ++ts;
+          did = true;
         }
-        tc_fence_after();
-        const uint32_t kb = smem_u32(smem + st * LY::STAGE);
-        const uint32_t khalf = (do_blk && t == n) ? (uint32_t)(KBR * TROWB) : (uint32_t)(TKT * TROWB);
-#pragma unroll
-        for (int h = 0; h < H; ++h)
-#pragma unroll
-          for (int ks = 0; ks < 4; ++ks)
-            umma_bf16(tmem_base + (uint32_t)((t & 1) * NT), smem_desc_sw128(kb + h * khalf + ks * 32),
-                      smem_desc_sw128(q0 + h * LY::QH + ks * 32), idesc_qk, (h | ks) != 0 ? 1u : 0u);
-        umma_commit(&s_full[t & 1]);
-        if (t >= 1 && !pv(t - 1)) {
+        if (did) {
+          t_last = global_timer_ns();
+        } else if (*abort_flag || global_timer_ns() - t_last > TC_WAIT_NS) {
           ok = false;
-          break;
         }
       }
-      if (ok && !pv(T - 1)) ok = false;
       if (!ok) {
         set_err(p.err, ERR_TIMEOUT);
         *abort_flag = 1;
@@ -430,25 +442,27 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ softmax
+    constexpr int HC = NT / 2;           // query-row columns of one softmax warp
     const int q = warp & 3;              // TMEM lane quarter this warp may access
     const int ew = warp - 2;
+    const int col0 = (ew >> 2) * HC;     // first of this warp's columns
     const int etid = tid - 64;
     const bool s_warp = true;            // every warp owns 32 keys (TMEM lanes)
     const int key = q * 32 + lane;
     if (p.kv_stable) {
       // warm L2 with the group's query rows before the producer's TMA
-      for (int e = etid; e < NR * (D * 2 / 128); e += 128) {
+      for (int e = etid; e < NR * (D * 2 / 128); e += TC_SOFT) {
         const int r = e / (D * 2 / 128), part_ = e % (D * 2 / 128);
         const int j = j0 + r / p.G, g = r % p.G;
         prefetch_l2(p.q + (((size_t)b * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D + part_ * 64);
       }
     }
-    float l_part[NT];
-    float mref[NT];                      // m_ref of every row (softmax lanes)
+    float l_part[HC];
+    float mref[HC];                      // m_ref of this warp's rows
 #pragma unroll
-    for (int r = 0; r < NT; ++r) {
-      l_part[r] = 0.f;
-      mref[r] = (r < NR) ? -INFINITY : INFINITY;
+    for (int i = 0; i < HC; ++i) {
+      l_part[i] = 0.f;
+      mref[i] = (col0 + i < NR) ? -INFINITY : INFINITY;
     }
     const float sc = p.scale_log2;
     bool aborted = false;
@@ -458,41 +472,41 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       const bool blk = do_blk && t == n;
       const bool okw = __all_sync(0xffffffffu, mbar_wait(&s_full[t & 1], (uint32_t)(t >> 1) & 1u, TC_WAIT_NS));
       tc_fence_after();
-      const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)((t & 1) * NT);
+      const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)((t & 1) * NT + col0);
       // cache keys below C are seen by every row; block key j < R by the
       // rows of block rows >= j (causal inside the block)
       const bool kvalid = blk ? (key < p.R) : ((t_begin + t) * TKT + key < C);
       // block key j is seen by row r iff j <= j0 + r / G, i.e. (j - j0) * G <= r
       // (causal), or by every row (full block)
       const int kg = p.block_full ? -1 : (key - j0) * p.G;
-      float x[NT];
+      float x[HC];
       float excess = -INFINITY;
       if (s_warp && okw) {
-        load_s<NT>(taddr, N, x);
+        load_s<HC>(taddr, N - col0, x);
         // x = score * log2(e) / sqrt(D) - m_ref; with m_ref unset (-inf) this
         // is +inf and forces the exact path below
         if (!blk) {
 #pragma unroll
-          for (int r = 0; r < NT; ++r) {
-            x[r] = kvalid ? fmaf(x[r], sc, -mref[r]) : -INFINITY;
-            excess = fmaxf(excess, x[r]);
+          for (int i = 0; i < HC; ++i) {
+            x[i] = kvalid ? fmaf(x[i], sc, -mref[i]) : -INFINITY;
+            excess = fmaxf(excess, x[i]);
           }
         } else {
 #pragma unroll
-          for (int r = 0; r < NT; ++r) {
-            x[r] = (kvalid && kg <= r) ? fmaf(x[r], sc, -mref[r]) : -INFINITY;
-            excess = fmaxf(excess, x[r]);
+          for (int i = 0; i < HC; ++i) {
+            x[i] = (kvalid && kg <= col0 + i) ? fmaf(x[i], sc, -mref[i]) : -INFINITY;
+            excess = fmaxf(excess, x[i]);
           }
         }
       }
       // vote: bit 0 = this warp saw a score above m_ref + 2^8, bit 1 = timeout
       const bool hi = __any_sync(0xffffffffu, excess > LAZY_LOG2);
-      if (lane == 0) votes[(t & 1) * 4 + ew] = (hi ? 1 : 0) | (okw ? 0 : 2);
+      if (lane == 0) votes[(t & 1) * 8 + ew] = (hi ? 1 : 0) | (okw ? 0 : 2);
       if (etid == 0) resc[t & 1] = 0;
-      named_bar_sync(1, 128);
+      named_bar_sync(1, TC_SOFT);
       int vote = 0;
 #pragma unroll
-      for (int w = 0; w < 4; ++w) vote |= votes[(t & 1) * 4 + w];
+      for (int w = 0; w < 8; ++w) vote |= votes[(t & 1) * 8 + w];
       if (vote & 2) {
         if (etid == 0) {
           set_err(p.err, ERR_TIMEOUT);
@@ -505,20 +519,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         // Exact path: absolute scaled scores of the tile, their column
         // maxima, the new references and the factors for what came before.
         if (s_warp) {
-          load_s<NT>(taddr, N, x);
+          load_s<HC>(taddr, N - col0, x);
 #pragma unroll
-          for (int r = 0; r < NT; ++r)
-            x[r] = (kvalid && (!blk || kg <= r)) ? x[r] * sc : -INFINITY;
+          for (int i = 0; i < HC; ++i)
+            x[i] = (kvalid && (!blk || kg <= col0 + i)) ? x[i] * sc : -INFINITY;
+          // column maxima over the warp's 32 keys (a 16-column half padded to 32)
+          float mx[32];
 #pragma unroll
-          for (int h32 = 0; h32 < NT / 32; ++h32) {
-            float mx[32];
-#pragma unroll
-            for (int i = 0; i < 32; ++i) mx[i] = x[h32 * 32 + i];
-            warp_col_reduce<32, true>(mx, lane);
-            red[q * NT + h32 * 32 + lane] = mx[0];
-          }
+          for (int i = 0; i < 32; ++i) mx[i] = (i < HC) ? x[i] : -INFINITY;
+          warp_col_reduce<32, true>(mx, lane);
+          if (lane < HC) red[q * NT + col0 + lane] = mx[0];
         }
-        named_bar_sync(1, 128);
+        named_bar_sync(1, TC_SOFT);
         if (etid < NT) {
           const int r = etid;
           const float mo = m_ref[r];
@@ -532,13 +544,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           alpha_s[r] = a;
           if (a < 1.f && t > 0) resc[t & 1] = 1;
         }
-        named_bar_sync(1, 128);
+        named_bar_sync(1, TC_SOFT);
         if (s_warp) {
 #pragma unroll
-          for (int r = 0; r < NT; ++r) {
-            mref[r] = m_ref[r];
-            l_part[r] *= alpha_s[r];
-            x[r] -= mref[r];
+          for (int i = 0; i < HC; ++i) {
+            mref[i] = m_ref[col0 + i];
+            l_part[i] *= alpha_s[col0 + i];
+            x[i] -= mref[i];
           }
         }
         if (resc[t & 1]) {
@@ -548,7 +560,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           if (okp && (H == 2 || q < 2)) {
             const uint32_t oaddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(2 * NT);
 #pragma unroll 1
-            for (int c = 0; c < NT / 16; ++c) {
+            for (int c = col0 / 16; c < (col0 + HC) / 16; ++c) {
               if (c * 16 < N) {
                 float o[16];
                 tmem_ld16_async(oaddr + c * 16, o);
@@ -570,13 +582,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         const int kk = key & 63;
         uint8_t* prow = sb + (key >> 6) * LY::PCS + (kk & 7) * 2;
 #pragma unroll
-        for (int c = 0; c < NT / 16; ++c) {
-          if (c * 16 < N) {
+        for (int c = 0; c < HC / 16; ++c) {
+          if (col0 + c * 16 < N) {
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
-              const int r = c * 16 + i;
-              const float pr = exp2_approx(x[r]);
-              l_part[r] += pr;
+              const int r = col0 + c * 16 + i;
+              const float pr = exp2_approx(x[c * 16 + i]);
+              l_part[c * 16 + i] += pr;
               *reinterpret_cast<__nv_bfloat16*>(prow + r * TROWB + (((kk >> 3) ^ (r & 7)) << 4)) =
                   __float2bfloat16_rn(pr);
             }
@@ -590,7 +602,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         const int rows = blk ? KBR : TKT;
         const int vhalf = rows * TROWB;
         uint8_t* vb = sb + LY::KVB;
-        for (int e = etid; e < (rows - vr) * H * 8; e += 128) {
+        for (int e = etid; e < (rows - vr) * H * 8; e += TC_SOFT) {
           const int row = vr + e / (H * 8), rem = e % (H * 8);
           *reinterpret_cast<uint4*>(vb + (rem / 8) * vhalf + row * TROWB + (rem % 8) * 16) =
               make_uint4(0u, 0u, 0u, 0u);
@@ -598,7 +610,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       }
       fence_proxy_async_smem();
       tc_fence_before();
-      named_bar_sync(1, 128);
+      named_bar_sync(1, TC_SOFT);
       if (etid == 0) {
         mbar_arrive(&p_full[t & 1]);
         mbar_arrive(&s_empty[t & 1]);
@@ -606,21 +618,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
     // Totals of the partial sums, and the end of the last P.V product.
     if (s_warp) {
+      float sm[32];
 #pragma unroll
-      for (int h32 = 0; h32 < NT / 32; ++h32) {
-        float sm[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) sm[i] = l_part[h32 * 32 + i];
-        warp_col_reduce<32, false>(sm, lane);
-        red[q * NT + h32 * 32 + lane] = sm[0];
-      }
+      for (int i = 0; i < 32; ++i) sm[i] = (i < HC) ? l_part[i] : 0.f;
+      warp_col_reduce<32, false>(sm, lane);
+      if (lane < HC) red[q * NT + col0 + lane] = sm[0];
     }
     if (T > 0 && !aborted) {
       const bool okp = __all_sync(0xffffffffu, mbar_wait(pv_done, (uint32_t)(T - 1) & 1u, TC_WAIT_NS));
       if (!okp && lane == 0) set_err(p.err, ERR_TIMEOUT);
     }
     tc_fence_after();
-    named_bar_sync(1, 128);
+    named_bar_sync(1, TC_SOFT);
     if (etid < NT)
       lsum[etid] = (T > 0 && !aborted)
                        ? (red[etid] + red[NT + etid]) + (red[2 * NT + etid] + red[3 * NT + etid])
@@ -641,10 +650,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   if (warp >= 2) {
     const int q = warp & 3;
     const int d = q * 32 + lane;
+    const int c0 = ((warp - 2) >> 2) * (NT / 32);    // this warp's half of the row chunks
     if (H == 2 || q < 2) {
       const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(2 * NT);
 #pragma unroll
-      for (int c = 0; c < NT / 16; ++c) {
+      for (int c = c0; c < c0 + NT / 32; ++c) {
         if (c * 16 < N) {
           float o[16];
           if (have) {
