@@ -6,16 +6,19 @@
 // (b, head, row group) form a thread-block cluster and merge their partial
 // softmax states through distributed shared memory, as in the mma.sync
 // variant.  Inside a CTA the roles are split by warp:
-//   warp 0      TMA producer: 128-key K/V tiles (one 2-D box per page and
+//   warps 0-2   TMA producers: 128-key K/V tiles (one 2-D box per page and
 //               128-byte half, so each tile lands as [half][128 keys][128 B],
 //               128B-swizzled) into a ring of stages, the query rows of the
-//               group once, the block's own K/V as a final tile;
-//   warp 1      MMA issuer (one thread):
+//               group once, the block's own K/V as a final tile.  A warp
+//               issues its bulk copies one after another, which holds one
+//               warp to about 45 GB/s of 2 KB boxes; three warps split each
+//               tile's 32 boxes;
+//   warp 3      MMA issuer (one thread):
 //                 S^T = K Q^T   (M = 128 keys, N = query rows, K = D),
 //                 O^T += V^T P^T (M = D, N = query rows, K = keys; V^T is
 //                               read MN-major straight from the V tile);
 //               S^T is double-buffered in TMEM, O^T accumulates in TMEM;
-//   warps 2-9   softmax: one thread per key (TMEM lane) turns a tile of S^T
+//   warps 4-11  softmax: one thread per key (TMEM lane) turns a tile of S^T
 //               into P^T (bf16, written over the tile's K, which the MMA no
 //               longer needs), rescales O^T when needed and reads it out at
 //               the end.  Two warps share each TMEM lane quarter and split
@@ -43,7 +46,10 @@ constexpr int TKT = 128;          // keys per cache tile (8 pages) = MMA M
 constexpr int TPPT = TKT / 16;    // pages per tile
 constexpr int TPAGE = 16;         // page size (fixed)
 constexpr int TROWB = 128;        // bytes of one swizzled smem row
-constexpr int TC_THREADS = 320;   // producer warp, MMA warp, 8 softmax warps
+constexpr int TC_PROD = 3;        // producer warps
+constexpr int TC_MMA_WARP = 3;    // MMA issuer warp
+constexpr int TC_SOFT0 = 4;       // first softmax warp
+constexpr int TC_THREADS = 384;   // producer warps, MMA warp, 8 softmax warps
 constexpr int TC_SOFT = 256;      // softmax threads
 constexpr float LAZY_LOG2 = 8.f;  // rescale only when a score exceeds m_ref by this (log2)
 constexpr uint64_t TC_WAIT_NS = 2000000000ull;
@@ -221,7 +227,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 
   if (tid == 0) {
     for (int s = 0; s < NS; ++s) {
-      mbar_init(&full[s], 1);
+      mbar_init(&full[s], TC_PROD);        // one arrival per producer warp
       mbar_init(&empty[s], 1);
     }
     mbar_init(q_full, 1);
@@ -236,7 +242,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     for (int i = 0; i < 20; ++i) votes[i] = 0;
     fence_barrier_init();
   }
-  if (warp == 1) {
+  if (warp == TC_MMA_WARP) {
     tmem_alloc(tmem_holder, LY::TCOLS);
     tmem_relinquish();
   }
@@ -274,9 +280,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   const int npages = (C + TPAGE - 1) / TPAGE;
   const int KBR = (p.R + 15) & ~15;                  // block keys padded to 16
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ producer
-    if (lane == 0) {
+  if (warp < TC_PROD) {
+    // ------------------------------------------------------------ producers
+    const int pw = warp;
+    constexpr int NBOX = 2 * H * TPPT;                  // boxes of a full tile
+    constexpr int BPW = (NBOX + TC_PROD - 1) / TC_PROD; // boxes per producer warp
+    const int e = pw * BPW + lane;                      // this lane's box
+    const bool mine = lane < BPW && e < NBOX;
+    if (pw == 0 && lane == 0) {
       tma_prefetch_desc(&map_kp);
       tma_prefetch_desc(&map_vp);
       tma_prefetch_desc(&map_q);
@@ -298,16 +309,20 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       }
       const int np = min(TPPT, npages - (t_begin + t) * TPPT);
       // box e: page e / (2H), tensor (e / H) & 1 (K, V), half e % H
-      const int pg = lane / (2 * H);
+      const int pg = e / (2 * H);
       int pgid = __shfl_sync(0xffffffffu, pid, (t & 3) * TPPT + (pg & 7));
-      if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)(np * 2 * H * TPAGE * TROWB));
+      if (lane == 0) {
+        // this warp's boxes within the tile's np pages
+        const int lo = pw * BPW, hi = min(NBOX, min(lo + BPW, np * 2 * H));
+        mbar_arrive_expect_tx(&full[st], (uint32_t)(max(0, hi - lo) * TPAGE * TROWB));
+      }
       __syncwarp();
-      if (lane < 2 * H * TPPT && pg < np) {
+      if (mine && pg < np) {
         if ((unsigned)pgid >= (unsigned)p.num_pages) {
           set_err(p.err, ERR_PAGE);
           pgid = 0;
         }
-        const int tensor = (lane / H) & 1, h = lane % H;
+        const int tensor = (e / H) & 1, h = e % H;
         tma_load_3d(smem_u32(sb + tensor * LY::KVB + h * (TKT * TROWB) + pg * (TPAGE * TROWB)),
                     tensor ? (const void*)&map_vp : (const void*)&map_kp, &full[st], 0,
                     (pgid * p.Hkv + kvh) * TPAGE, h, pol);
@@ -325,7 +340,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       issue_cache(t);
       ++issued;
     }
-    if (pre == NS && n > NS) {
+    if (pw == 0 && pre == NS && n > NS) {
       // The ring is full: pull the next tile's pages into L2.
       const int e = NS * TPPT + (lane >> 1);
       const int pg = __shfl_sync(0xffffffffu, pid, e & 31);
@@ -334,8 +349,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           tma_prefetch_l2_3d((lane & 1) ? (const void*)&map_vp : (const void*)&map_kp, 0,
                              (pg * p.Hkv + kvh) * TPAGE, h);
     }
-    if (p.kv_stable) griddep_wait();     // the query rows and the block K/V come from it
-    if (T > 0 && lane == 0) {
+    // the query rows and the block K/V come from the previous kernel; the
+    // other producers read only the (stable) cache
+    if (p.kv_stable && pw == 0) griddep_wait();
+    if (T > 0 && pw == 0 && lane == 0) {
       mbar_arrive_expect_tx(q_full, (uint32_t)(H * qrows * TROWB));
       for (int h = 0; h < H; ++h)
         tma_load_4d(smem_u32(qs + h * LY::QH), &map_q, q_full, 0, kvh * p.G, b * p.R + j0, h, pol);
@@ -353,12 +370,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       if (wait_slot(t)) {
         const int st = t % NS;
         uint8_t* sb = smem + st * LY::STAGE;
-        if (lane == 0) {
+        if (pw == 0 && lane == 0) {
           // one box per tensor: KBR rows from block row 0 of this head, all
           // halves, landing as [half][KBR rows][128 B]
           mbar_arrive_expect_tx(&full[st], (uint32_t)(2 * H * KBR * TROWB));
           tma_load_4d(smem_u32(sb), &map_kb, &full[st], 0, b * p.R, 0, kvh, pol);
           tma_load_4d(smem_u32(sb + LY::KVB), &map_vb, &full[st], 0, b * p.R, 0, kvh, pol);
+        } else if (lane == 0) {
+          mbar_arrive(&full[st]);
         }
         ++issued;
       } else {
@@ -369,8 +388,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       set_err(p.err, ERR_TIMEOUT);
       *abort_flag = 1;
     }
-    if (lane == 0) *n_issued = issued;
-  } else if (warp == 1) {
+    if (pw == 0 && lane == 0) *n_issued = issued;
+  } else if (warp == TC_MMA_WARP) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && T > 0) {
       const uint32_t idesc_qk = idesc_bf16_f32(128, N);
@@ -444,9 +463,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     // ------------------------------------------------------------ softmax
     constexpr int HC = NT / 2;           // query-row columns of one softmax warp
     const int q = warp & 3;              // TMEM lane quarter this warp may access
-    const int ew = warp - 2;
+    const int ew = warp - TC_SOFT0;
     const int col0 = (ew >> 2) * HC;     // first of this warp's columns
-    const int etid = tid - 64;
+    const int etid = tid - TC_SOFT0 * 32;
     const bool s_warp = true;            // every warp owns 32 keys (TMEM lanes)
     const int key = q * 32 + lane;
     if (p.kv_stable) {
@@ -647,10 +666,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   }
   float* part = reinterpret_cast<float*>(smem + LY::PART);
   const bool have = T > 0 && !*abort_flag;
-  if (warp >= 2) {
+  if (warp >= TC_SOFT0) {
     const int q = warp & 3;
     const int d = q * 32 + lane;
-    const int c0 = ((warp - 2) >> 2) * (NT / 32);    // this warp's half of the row chunks
+    const int c0 = ((warp - TC_SOFT0) >> 2) * (NT / 32);   // this warp's half of the row chunks
     if (H == 2 || q < 2) {
       const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(2 * NT);
 #pragma unroll
@@ -749,7 +768,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (warp == 1) {
+  if (warp == TC_MMA_WARP) {
     __syncwarp();
     tmem_dealloc(tmem_base, LY::TCOLS);
   }
