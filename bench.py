@@ -457,7 +457,7 @@ def main():
         achieved = lmhead_flops(cfg) / (lm_ms * 1e-3) / 1e12
         roof = {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": tflops_peak,
                 "unit": "TFLOP/s", "frac": achieved / tflops_peak, "traffic": None}
-    roof["peak_source"] = f"{pk_kind} ({PEAKS_FILE if pk_kind == 'measured' else 'recipe fallback'})"
+    roof["peak_source"] = f"{pk_kind} ({'MEASURED_PEAKS.json' if pk_kind == 'measured' else 'recipe fallback'})"
     if roof["unit"] == "GB/s":
         roof["frac_of_spec_8tbs"] = roof["achieved"] / 7900.0   # nominal HBM3e, for context
     traffic = TRAFFIC.get((cfg.name, dom))
@@ -509,8 +509,9 @@ def main():
 # (profiles/), keyed by (workload, kernel); an entry is removed when its
 # kernel changes after the capture.
 TRAFFIC = {
-    ("qwen3_8b_b1", "verify_attn"): 16915200.0,
-    ("qwen3_8b_b1", "lmhead_argmax_features"): 1247979104.0,
+    ("qwen3_8b_b1", "verify_attn"): 16918016.0,
+    ("qwen3_8b_b1", "lmhead_argmax_features"): 1247823104.0,
+    ("qwen3_32b_b32", "verify_attn"): 1362588416.0,
 }
 
 
