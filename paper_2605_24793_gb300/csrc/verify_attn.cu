@@ -186,16 +186,16 @@ CS_DEV void attend(uint32_t sk, uint32_t sv, uint32_t group_bytes, uint32_t half
 // 168).  With more block keys the shared memory allows one CTA per SM, and
 // it keeps its registers (no spills).
 template <int D, int MT, int WK, int GEN>
-__global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 32,
-                                  MT >= 4 && GEN < 2 ? 2 : 0)
+__global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 64,
+                                  MT >= 4 && GEN < 2 ? 2 : (GEN == 2 ? 1 : 0))
     verify_attn_kernel(const __grid_constant__ CUtensorMap map_kp,
                        const __grid_constant__ CUtensorMap map_vp,
                        const __grid_constant__ CUtensorMap map_kb,
                        const __grid_constant__ CUtensorMap map_vb, const AttnParams p) {
   using LY = Layout<D, MT, WK>;
-  constexpr int NWARPS = MT * WK;        // consumer warps; warp NWARPS issues the loads
+  constexpr int NWARPS = MT * WK;        // consumer warps; warps NWARPS (K) and NWARPS+1 (V) issue the loads
   constexpr int NTC = NWARPS * 32;
-  constexpr int NTT = NTC + 32;
+  constexpr int NTT = NTC + 64;
   constexpr int KW = KT / WK;            // cache keys of a tile handled by one warp
   constexpr int H = LY::H;
   constexpr int NRP = LY::NRP;
@@ -221,7 +221,7 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 32,
 
   if (tid == 0) {
     for (int s2 = 0; s2 < NSTAGE; ++s2) {
-      mbar_init(&full[s2], 1);
+      mbar_init(&full[s2], 2);           // the K and the V producer
       mbar_init(&empty[s2], NWARPS);
     }
     mbar_init(blk_full, 1);
@@ -259,8 +259,11 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 32,
   const int wr = warp / WK, wk = warp % WK;
   const int r0 = wr * 16 + g_row, r1 = r0 + 8;
 
-  if (warp == NWARPS) {
-    // ---------------------------------------------------------- producer warp
+  if (warp >= NWARPS) {
+    // ---------------------------------------------------------- producer warps
+    // A warp's bulk copies are processed one after another; two warps (one
+    // for K, one for V) double the rate at which a CTA can pull tiles.
+    const int tensor = warp - NWARPS;    // 0: K, 1: V
     if (lane == 0) {
       tma_prefetch_desc(&map_kp);
       tma_prefetch_desc(&map_vp);
@@ -276,7 +279,7 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 32,
         waited = true;
       }
     }
-    if (do_blk && lane == 0) {
+    if (do_blk && tensor == 0 && lane == 0) {
       // one box per tensor: KBR rows from block row 0 of this head, both halves
       // (rows past R belong to the next sequence or are zero-filled; masked)
       mbar_arrive_expect_tx(blk_full, (uint32_t)(H * 2 * ROWB * KBR));   // KBR-row boxes
@@ -297,28 +300,27 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 32,
       uint8_t* kb = smem + st * LY::STAGE;
       {
         const int np = min(4, npages - (t_begin + vt) * 4);
-        // lanes 0..7: page lane/2 of the tile, K (even lane) or V (odd lane)
-        int pgid = __shfl_sync(0xffffffffu, pid, (vt & 7) * 4 + ((lane >> 1) & 3));
-        if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)(np * 2 * LY::PAGEB));
+        // lanes 0..3: page `lane` of the tile, this warp's tensor
+        int pgid = __shfl_sync(0xffffffffu, pid, (vt & 7) * 4 + (lane & 3));
+        if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)(np * LY::PAGEB));
         __syncwarp();
-        if (lane < 2 * np) {
+        if (lane < np) {
           if ((unsigned)pgid >= (unsigned)p.num_pages) {
             set_err(p.err, ERR_PAGE);
             pgid = 0;
           }
           const int y = (pgid * p.Hkv + kvh) * PAGE;
-          const int pg = lane >> 1;
-          tma_load_3d(smem_u32(kb + (lane & 1) * LY::KV + pg * LY::PAGEB), (lane & 1) ? (const void*)&map_vp : (const void*)&map_kp,
-                      &full[st], 0, y, 0, pol);
+          tma_load_3d(smem_u32(kb + tensor * LY::KV + lane * LY::PAGEB),
+                      tensor ? (const void*)&map_vp : (const void*)&map_kp, &full[st], 0, y, 0, pol);
         }
       }
       if (vt == NSTAGE - 1) {
         // The ring is full: pull the next two tiles' pages into L2 so their
         // loads, issued once stages free up, skip most of the HBM latency.
-        const int e = NSTAGE * 4 + (lane >> 1);                  // lanes 0..15: 8 pages, K and V
+        const int e = NSTAGE * 4 + lane;                         // lanes 0..7: 8 pages
         const int pg = __shfl_sync(0xffffffffu, pid, e & 31);
-        if (lane < 16 && e < my_pages && (unsigned)pg < (unsigned)p.num_pages)
-          tma_prefetch_l2_3d((lane & 1) ? (const void*)&map_vp : (const void*)&map_kp, 0,
+        if (lane < 8 && e < my_pages && (unsigned)pg < (unsigned)p.num_pages)
+          tma_prefetch_l2_3d(tensor ? (const void*)&map_vp : (const void*)&map_kp, 0,
                              (pg * p.Hkv + kvh) * PAGE, 0);
       }
       __syncwarp();
@@ -597,7 +599,7 @@ cudaError_t launch_t(const CUtensorMap* maps, const AttnParams& p, int S, int B,
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(S, Hkv * p.RG, B);
-  cfg.blockDim = dim3(MT * WK * 32 + 32, 1, 1);
+  cfg.blockDim = dim3(MT * WK * 32 + 64, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
@@ -629,7 +631,7 @@ int max_cluster_t(int S, int Hkv, int B, int kbr) {
   cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(S, Hkv, B);
-  cfg.blockDim = dim3(MT * WK * 32 + 32, 1, 1);
+  cfg.blockDim = dim3(MT * WK * 32 + 64, 1, 1);
   cfg.dynamicSmemBytes = LY::total(kbr) + 1024;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
