@@ -272,20 +272,27 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 64,
     // (running side by side) keep it in L2 for the siblings
     const uint64_t pol = p.RG > 1 ? l2_policy_evict_normal() : l2_policy_evict_first();
     bool waited = !p.kv_stable;
-    if (do_blk && p.R > 0) {
-      // the block K/V is written by the previous kernel: wait first
+    // The block K/V is written by the previous kernel: the V producer of the
+    // CTA that owns the block fills its ring with cache tiles first (they
+    // may stream early), then waits for that kernel and loads the block.
+    const bool blk_here = do_blk && tensor == 1;
+    const int blk_after = min(nv, NSTAGE);   // cache tiles issued before the block
+    auto issue_block = [&]() {
       if (!waited) {
         griddep_wait();
         waited = true;
       }
-    }
-    if (do_blk && tensor == 0 && lane == 0) {
-      // one box per tensor: KBR rows from block row 0 of this head, both halves
-      // (rows past R belong to the next sequence or are zero-filled; masked)
-      mbar_arrive_expect_tx(blk_full, (uint32_t)(H * 2 * ROWB * KBR));   // KBR-row boxes
-      tma_load_4d(smem_u32(blk_k), &map_kb, blk_full, 0, b * p.R, 0, kvh, pol);
-      tma_load_4d(smem_u32(blk_v), &map_vb, blk_full, 0, b * p.R, 0, kvh, pol);
-    }
+      if (lane == 0) {
+        // one box per tensor: KBR rows from block row 0 of this head, both
+        // halves (rows past R belong to the next sequence or are zero-filled;
+        // masked)
+        mbar_arrive_expect_tx(blk_full, (uint32_t)(H * 2 * ROWB * KBR));   // KBR-row boxes
+        tma_load_4d(smem_u32(blk_k), &map_kb, blk_full, 0, b * p.R, 0, kvh, pol);
+        tma_load_4d(smem_u32(blk_v), &map_vb, blk_full, 0, b * p.R, 0, kvh, pol);
+      }
+      __syncwarp();
+    };
+    if (blk_here && blk_after == 0) issue_block();
     const int* ptab = p.page_table + (size_t)b * p.max_pages + (size_t)t_begin * 4;
     const int my_pages = min(n * 4, npages - t_begin * 4);   // page-table entries of this CTA
     int pid = 0;
@@ -324,6 +331,7 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 64,
                              (pg * p.Hkv + kvh) * PAGE, 0);
       }
       __syncwarp();
+      if (blk_here && vt == blk_after - 1) issue_block();
     }
     if (!waited) griddep_wait();
   } else {
