@@ -30,16 +30,18 @@ __global__ void __launch_bounds__(WARPS * 32)
   extern __shared__ float sm[];            // w1 [H][8], b1 [H], w2 [H] when mode == 0
   __shared__ float feat[WARPS][32][NF];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  griddep_wait();
-  griddep_launch_dependents();
+  // The MLP weights do not come from the previous kernel: stage them while
+  // it finishes, then wait for its statistics.
   if (mode == 0) {
     for (int e = threadIdx.x; e < H * NF; e += blockDim.x) sm[e] = w1[e];
     for (int e = threadIdx.x; e < H; e += blockDim.x) {
       sm[H * NF + e] = b1[e];
       sm[H * NF + H + e] = w2[e];
     }
-    __syncthreads();
   }
+  griddep_wait();
+  griddep_launch_dependents();
+  if (mode == 0) __syncthreads();
   const int b = blockIdx.x * WARPS + warp;
   if (b >= B) return;
 

@@ -278,7 +278,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
-  griddep_wait();                        // hidden rows may come from the previous kernel
+  // The hidden rows may come from the previous kernel (the producer waits
+  // for it after streaming its first W stages, which do not).
+  if (warp != 0) griddep_wait();
   uint32_t seed_lo = 0, seed_hi = 0;
   if (warp >= 2) {
     if (KEYED) {
@@ -305,17 +307,34 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       uint32_t phase = 0;
       uint32_t issued_mask = 0, issued_parity = 0;   // last load per stage (stages <= 16)
       bool ok = true;
+      // The first ring's worth of W stages streams before the wait for the
+      // previous kernel; their hidden-row boxes follow it.
+      const int my_tiles = blockIdx.x < p.num_tiles ? (p.num_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
+      const int npre = min(p.stages, my_tiles * kblocks);
+      for (int i = 0; i < npre; ++i) {
+        const int tile = blockIdx.x + (i / kblocks) * gridDim.x, kb = i % kblocks;
+        mbar_arrive_expect_tx(&full[i], (uint32_t)A_BYTES + b_bytes);
+        tma_load_2d(smem_u32(smem + L.a_off + (uint32_t)i * A_BYTES), &tmap_w, &full[i], kb * BK,
+                    tile * BM, pol_w);
+      }
+      griddep_wait();
+      for (int i = 0; i < npre; ++i)
+        tma_load_2d(smem_u32(smem + L.b_off + (uint32_t)i * b_bytes), &tmap_h, &full[i],
+                    (i % kblocks) * BK, p.row0, pol_h);
+      int li = 0;                        // loads so far, in (tile, k-block) order
       for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
-        for (int kb = 0; kb < kblocks; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, WAIT_NS) || *abort_flag) {
-            ok = false;
-            break;
+        for (int kb = 0; kb < kblocks; ++kb, ++li) {
+          if (li >= npre) {
+            if (!mbar_wait(&empty[stage], phase ^ 1u, WAIT_NS) || *abort_flag) {
+              ok = false;
+              break;
+            }
+            const uint32_t sa = smem_u32(smem + L.a_off + (uint32_t)stage * A_BYTES);
+            const uint32_t sb = smem_u32(smem + L.b_off + (uint32_t)stage * b_bytes);
+            mbar_arrive_expect_tx(&full[stage], (uint32_t)A_BYTES + b_bytes);
+            tma_load_2d(sa, &tmap_w, &full[stage], kb * BK, tile * BM, pol_w);
+            tma_load_2d(sb, &tmap_h, &full[stage], kb * BK, p.row0, pol_h);
           }
-          const uint32_t sa = smem_u32(smem + L.a_off + (uint32_t)stage * A_BYTES);
-          const uint32_t sb = smem_u32(smem + L.b_off + (uint32_t)stage * b_bytes);
-          mbar_arrive_expect_tx(&full[stage], (uint32_t)A_BYTES + b_bytes);
-          tma_load_2d(sa, &tmap_w, &full[stage], kb * BK, tile * BM, pol_w);
-          tma_load_2d(sb, &tmap_h, &full[stage], kb * BK, p.row0, pol_h);
           issued_mask |= 1u << stage;
           issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
           if (++stage == p.stages) {
