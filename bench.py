@@ -509,8 +509,8 @@ def main():
 # (profiles/), keyed by (workload, kernel); an entry is removed when its
 # kernel changes after the capture.
 TRAFFIC = {
-    ("qwen3_8b_b1", "verify_attn"): 16918016.0,
-    ("qwen3_8b_b1", "lmhead_argmax_features"): 1247823104.0,
+    ("qwen3_8b_b1", "verify_attn"): 16917504.0,
+    ("qwen3_8b_b1", "lmhead_argmax_features"): 1247705088.0,
     ("qwen3_32b_b32", "verify_attn"): 1362588416.0,
 }
 
