@@ -692,12 +692,15 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
     pl.jbq = jbq;
     pl.rg = (R + pl.jb - 1) / pl.jb;
     pl.nt = ((G * pl.jbq + 15) / 16 * 16) <= 32 ? 32 : 64;
-    // 128-key tiles; about one CTA per SM (a stage ring of 96-192 KB), at
-    // least two tiles per CTA, no CTA with more than 64 tiles (long
-    // sequences split, so that uneven contexts balance over the waves).
+    // 128-key tiles; one CTA per SM (a stage ring of 96-192 KB); about three
+    // waves of CTAs or more (finer work balances the tail: measured on the
+    // Qwen3-32B batch-32 and Qwen3-8B batch-16 K = 25 workloads, 256 units
+    // ran best with 2 splits, ahead of 1 and 4), at least two tiles per CTA,
+    // no CTA with more than 64 tiles (long sequences split, so that uneven
+    // contexts balance over the waves).
     const int tiles_tc = (max_ctx + 127) / 128;
     pl.units = (long long)B * Hkv * pl.rg;
-    const long long wave_tc = ((long long)num_sms + pl.units - 1) / (pl.units > 0 ? pl.units : 1);
+    const long long wave_tc = (3LL * num_sms + pl.units - 1) / (pl.units > 0 ? pl.units : 1);
     const long long len_tc = (tiles_tc + 63) / 64;
     const long long want_tc = wave_tc > len_tc ? wave_tc : len_tc;
     while (S < 16 && S < want_tc && (S * 2) * 2 <= tiles_tc) S *= 2;

@@ -127,7 +127,7 @@ def test_verify_attention_tcgen05_matches_oracle(case):
 # distributed shared memory, with most sequences far shorter than the split.
 ATTN_TC_SPLIT_CASES = [
     # B, R, Hq, Hkv, D, contexts, shuffled, expected splits
-    (20, 8, 64, 8, 128, [9000] + _ctx(19, 8), True, 2),
+    (40, 8, 64, 8, 128, [9000] + _ctx(39, 8), True, 2),
     (20, 16, 32, 8, 128, [20000, 3000] + _ctx(18, 9), True, 4),
     (20, 8, 64, 8, 128, [33000, 9000] + _ctx(18, 10), False, 8),
 ]
