@@ -69,6 +69,12 @@ typedef enum {
 /* Human-readable name of a cospec_status value (static string). */
 COSPEC_API const char* cospec_status_string(int status);
 
+/* Name of the CUDA runtime error behind the last COSPEC_ERR_CUDA that a call
+ * made on this host thread returned ("cudaSuccess" when there was none;
+ * static string).  Lets a caller tell, e.g., an invalid stream from an
+ * unsupported launch configuration. */
+COSPEC_API const char* cospec_last_cuda_error(void);
+
 /* Reads the device error word into *flags, then clears it.  Synchronises
  * `stream` first, so every kernel queued before is included.  Returns
  * COSPEC_OK, or COSPEC_ERR_DEVICE_CHECK when *flags != 0. */

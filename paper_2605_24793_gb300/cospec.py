@@ -19,7 +19,7 @@ LIB_PATH = os.path.join(_HERE, "libcospec.so")
 POLICY_MLP, POLICY_TARGET, POLICY_DRAFT = 0, 1, 2
 DEVERR_PAGE, DEVERR_CTX, DEVERR_TOKEN, DEVERR_TIMEOUT, DEVERR_OFFSETS = 1, 2, 4, 8, 16
 
-EXPORTED = ("cospec_status_string", "cospec_get_device_error", "cospec_num_sms",
+EXPORTED = ("cospec_status_string", "cospec_last_cuda_error", "cospec_get_device_error", "cospec_num_sms",
             "cospec_verify_attn", "cospec_lmhead_workspace", "cospec_lmhead_argmax_features",
             "cospec_arbitrate", "cospec_accept_commit", "cospec_lmhead_argmax_features_noalloc",
             "cospec_lmhead_sample_features", "cospec_verify_attn_plan", "cospec_rl_workspace",
@@ -68,6 +68,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib = ctypes.CDLL(path)
     sig = {
         "cospec_status_string": (ctypes.c_char_p, [_i]),
+        "cospec_last_cuda_error": (ctypes.c_char_p, []),
         "cospec_get_device_error": (_i, [ctypes.POINTER(_i), _vp]),
         "cospec_num_sms": (_i, []),
         "cospec_verify_attn": (_i, [_PDIMS, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
@@ -95,7 +96,10 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
 
 def _check(status: int) -> None:
     if status != 0:
-        msg = load_library().cospec_status_string(status).decode()
+        lib = load_library()
+        msg = lib.cospec_status_string(status).decode()
+        if status == -4:   # COSPEC_ERR_CUDA: name the runtime error behind it
+            msg += f": {lib.cospec_last_cuda_error().decode()}"
         raise CospecError(f"cospec call failed: {msg} ({status})")
 
 

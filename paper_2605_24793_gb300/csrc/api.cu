@@ -4,6 +4,9 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <atomic>
+#include <mutex>
+
 #include "../../include/cospec.h"
 #include "cospec_internal.h"
 
@@ -13,14 +16,25 @@ namespace {
 __device__ int g_error_word;   // one per device context; bits COSPEC_DEVERR_*
 
 constexpr int MAX_DEV = 64;
-int g_num_sms[MAX_DEV] = {0};
-int* g_err_ptr[MAX_DEV] = {nullptr};
+// Lazily filled per-device values; a race between host threads only
+// repeats the same query.
+std::atomic<int> g_num_sms[MAX_DEV];
+std::atomic<int*> g_err_ptr[MAX_DEV];
+std::mutex g_limits_mutex;
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// The calling thread's device, with its primary context made current the
+// first time (a host thread that has made no CUDA call yet has no current
+// context, and the tensor-map encoder needs one).
 int current_device() {
+  static thread_local int bound = -1;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return -1;
+  if (bound != dev) {
+    if (cudaSetDevice(dev) != cudaSuccess) return -1;
+    bound = dev;
+  }
   return dev;
 }
 }  // namespace
@@ -28,23 +42,47 @@ int current_device() {
 int device_num_sms() {
   const int dev = current_device();
   if (dev < 0 || dev >= MAX_DEV) return 0;
-  if (g_num_sms[dev] == 0) {
-    int n = 0;
+  int n = g_num_sms[dev].load(std::memory_order_relaxed);
+  if (n == 0) {
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    g_num_sms[dev] = n;
+    g_num_sms[dev].store(n, std::memory_order_relaxed);
   }
-  return g_num_sms[dev];
+  return n;
 }
 
 int* device_error_word() {
   const int dev = current_device();
   if (dev < 0 || dev >= MAX_DEV) return nullptr;
-  if (!g_err_ptr[dev]) {
+  int* ptr = g_err_ptr[dev].load(std::memory_order_acquire);
+  if (!ptr) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
-    g_err_ptr[dev] = static_cast<int*>(p);
+    ptr = static_cast<int*>(p);
+    g_err_ptr[dev].store(ptr, std::memory_order_release);
   }
-  return g_err_ptr[dev];
+  return ptr;
+}
+
+cudaError_t ensure_kernel_limits(const void* kern, KernelLimits& lim, size_t smem_bytes,
+                                 bool cluster) {
+  const int dev = current_device();
+  if (dev < 0 || dev >= KL_MAX_DEV) return cudaErrorInvalidDevice;
+  if (lim.smem[dev].load(std::memory_order_acquire) >= smem_bytes &&
+      (!cluster || lim.cluster[dev].load(std::memory_order_acquire)))
+    return cudaSuccess;
+  std::lock_guard<std::mutex> guard(g_limits_mutex);
+  if (lim.smem[dev].load(std::memory_order_relaxed) < smem_bytes) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes);
+    if (e != cudaSuccess) return e;
+    lim.smem[dev].store(smem_bytes, std::memory_order_release);
+  }
+  if (cluster && !lim.cluster[dev].load(std::memory_order_relaxed)) {
+    const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+    lim.cluster[dev].store(true, std::memory_order_release);
+  }
+  return cudaSuccess;
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -54,7 +92,8 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
 
 bool encode_tensor_map_bf16(void* map, const void* base, int rank, const uint64_t* dims,
                             const uint64_t* strides, const uint32_t* box) {
-  static EncodeTiledFn fn = nullptr;
+  static std::atomic<EncodeTiledFn> fn_cache{nullptr};
+  EncodeTiledFn fn = fn_cache.load(std::memory_order_acquire);
   if (!fn) {
     void* ptr = nullptr;
     cudaDriverEntryPointQueryResult q;
@@ -63,6 +102,7 @@ bool encode_tensor_map_bf16(void* map, const void* base, int rank, const uint64_
         q != cudaDriverEntryPointSuccess)
       return false;
     fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    fn_cache.store(fn, std::memory_order_release);
   }
   if (rank < 1 || rank > 5) return false;
   cuuint64_t d[5];
@@ -89,7 +129,14 @@ using namespace cospec;
     if (!(cond)) return COSPEC_ERR_INVALID_ARG; \
   } while (0)
 
-static int from_cuda(cudaError_t e) { return e == cudaSuccess ? COSPEC_OK : COSPEC_ERR_CUDA; }
+// The CUDA error behind this host thread's last COSPEC_ERR_CUDA.
+static thread_local cudaError_t t_last_cuda_error = cudaSuccess;
+
+static int from_cuda(cudaError_t e) {
+  if (e == cudaSuccess) return COSPEC_OK;
+  t_last_cuda_error = e;
+  return COSPEC_ERR_CUDA;
+}
 
 extern "C" {
 
@@ -106,6 +153,8 @@ COSPEC_API const char* cospec_status_string(int status) {
 }
 
 COSPEC_API int cospec_num_sms(void) { return device_num_sms(); }
+
+COSPEC_API const char* cospec_last_cuda_error(void) { return cudaGetErrorName(t_last_cuda_error); }
 
 COSPEC_API int cospec_get_device_error(int* flags, void* stream) {
   CS_CHECK_ARG(flags != nullptr);
@@ -143,7 +192,7 @@ static int check_attn_dims(const cospec_attn_dims* d) {
 // memory, not on the grid).
 static long long resident_clusters(int D, const AttnPlan& pl, int S, int Hkv, int B, int R) {
   // [dev][D==128][variant][block keys / 16 - 1][log2 S]: count + 1 (0: not yet queried)
-  static int cache[MAX_DEV][2][6][4][5];
+  static std::atomic<int> cache[MAX_DEV][2][6][4][5];
   const int kbr = (R + 15) & ~15;
   int dev = 0;
   cudaGetDevice(&dev);
@@ -152,10 +201,13 @@ static long long resident_clusters(int D, const AttnPlan& pl, int S, int Hkv, in
                               : (pl.mt == 1 ? 0 : pl.mt == 2 ? 1 : pl.mt == 4 ? 2 : 3);
   int ls = 0;
   while ((1 << ls) < S) ++ls;
-  int& c = cache[dev < MAX_DEV ? dev : MAX_DEV - 1][di][mi][kbr / 16 - 1][ls];
-  if (c == 0)
+  std::atomic<int>& slot = cache[dev < MAX_DEV ? dev : MAX_DEV - 1][di][mi][kbr / 16 - 1][ls];
+  int c = slot.load(std::memory_order_relaxed);
+  if (c == 0) {
     c = 1 + (pl.kind == 1 ? attn_tc_max_active_clusters(D, pl.nt, S, Hkv, B, pl.rg)
                           : attn_max_active_clusters(D, pl.mt, pl.wk, S, Hkv, B, kbr));
+    slot.store(c, std::memory_order_relaxed);
+  }
   return c - 1;
 }
 

@@ -4,6 +4,8 @@
 
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
+
+#include <atomic>
 #include <functional>
 #include <stddef.h>
 #include <stdint.h>
@@ -31,6 +33,20 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
 
 int device_num_sms();
 int* device_error_word();  // device address of the error word of the current device
+
+// Per-device record of the limits already set on one kernel.
+constexpr int KL_MAX_DEV = 64;
+struct KernelLimits {
+  std::atomic<size_t> smem[KL_MAX_DEV];   // dynamic shared-memory limit set so far
+  std::atomic<bool> cluster[KL_MAX_DEV];  // non-portable cluster sizes allowed
+};
+// Raise `kern`'s dynamic shared-memory limit on the current device to at
+// least `smem_bytes` (never lowering it, so graphs captured earlier stay
+// launchable) and, with `cluster`, allow non-portable cluster sizes.  Calls
+// from several host threads are serialised; later calls that need nothing
+// new only read `lim`.
+cudaError_t ensure_kernel_limits(const void* kern, KernelLimits& lim, size_t smem_bytes,
+                                 bool cluster);
 
 // cuTensorMapEncodeTiled for a bf16 tensor (rank 1..5, innermost first),
 // 128-byte swizzle, zero fill out of bounds.  dims/box in elements, strides

@@ -32,6 +32,8 @@
 #include <math.h>
 
 #include "../../include/cospec.h"
+#include <atomic>
+
 #include "cospec_device.cuh"
 #include "cospec_internal.h"
 
@@ -547,6 +549,13 @@ bool make_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, 
 
 }  // namespace
 
+// Limits already set on each variant of the kernel.
+template <bool KEYED>
+KernelLimits& lm_limits() {
+  static KernelLimits lim;
+  return lim;
+}
+
 LmheadPlan plan_lmhead(int M, int d, int V, int num_sms) {
   LmheadPlan pl{};
   const int rows = M < MAX_ROWS ? M : MAX_ROWS;
@@ -579,18 +588,11 @@ cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
   if (!make_map(&map_w, w, (uint64_t)V, (uint64_t)d, BM)) return cudaErrorInvalidValue;
   if (!make_map(&map_h, hidden, (uint64_t)M, (uint64_t)d, (uint32_t)pl.n_mma))
     return cudaErrorInvalidValue;
-  static bool configured[2][64] = {{false}};
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev < 64 && !configured[keyed][dev]) {
-    cudaError_t e = keyed ? cudaFuncSetAttribute(lmhead_kernel<true>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 227 * 1024)
-                          : cudaFuncSetAttribute(lmhead_kernel<false>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 227 * 1024);
+  {
+    const cudaError_t e =
+        keyed ? ensure_kernel_limits((const void*)lmhead_kernel<true>, lm_limits<true>(), 227 * 1024, false)
+              : ensure_kernel_limits((const void*)lmhead_kernel<false>, lm_limits<false>(), 227 * 1024, false);
     if (e != cudaSuccess) return e;
-    configured[keyed][dev] = true;
   }
   float4* part = static_cast<float4*>(ws);
   int* part_idx = reinterpret_cast<int*>(part + (size_t)1024 * MAX_ROWS);
@@ -659,17 +661,17 @@ constexpr size_t NOALLOC_ENTRIES = (size_t)NOALLOC_MAX_CTAS * MAX_ROWS;
 // [NOALLOC_ENTRIES] float4 (m, second, s, t) then [NOALLOC_ENTRIES] int (argmax)
 static __device__ __align__(256) unsigned char g_lmhead_scratch[NOALLOC_ENTRIES * (sizeof(float4) + sizeof(int))];
 
-void* g_scratch_addr[64] = {nullptr};
+std::atomic<void*> g_scratch_addr[64];   // per device; a race only repeats the lookup
 
 void* scratch_address() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-  if (!g_scratch_addr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_lmhead_scratch) != cudaSuccess) return nullptr;
-    g_scratch_addr[dev] = p;
+  void* addr = g_scratch_addr[dev].load(std::memory_order_acquire);
+  if (!addr) {
+    if (cudaGetSymbolAddress(&addr, g_lmhead_scratch) != cudaSuccess) return nullptr;
+    g_scratch_addr[dev].store(addr, std::memory_order_release);
   }
-  return g_scratch_addr[dev];
+  return addr;
 }
 
 }  // namespace
@@ -701,15 +703,9 @@ extern "C" COSPEC_API int cospec_lmhead_argmax_features_noalloc(
   if (!make_map(&map_w, w, (uint64_t)V, (uint64_t)d, BM) ||
       !make_map(&map_h, hidden, (uint64_t)M, (uint64_t)d, (uint32_t)pl.n_mma))
     return COSPEC_ERR_CUDA;
-  static bool configured[64] = {false};
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev < 64 && !configured[dev]) {
-    if (cudaFuncSetAttribute(lmhead_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             227 * 1024) != cudaSuccess)
-      return COSPEC_ERR_CUDA;
-    configured[dev] = true;
-  }
+  if (ensure_kernel_limits((const void*)lmhead_kernel<false>, lm_limits<false>(), 227 * 1024, false) !=
+      cudaSuccess)
+    return COSPEC_ERR_CUDA;
   uint32_t tmem_cols = 32;
   while (tmem_cols < (uint32_t)(2 * pl.n_mma)) tmem_cols <<= 1;
   // Each pass overwrites every scratch entry its merge kernel reads, so the

@@ -583,28 +583,21 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 64,
 }
 
 
+// Limits already set on each instantiation of the kernel.
+template <int D, int MT, int WK, int GEN>
+KernelLimits& attn_limits() {
+  static KernelLimits lim;
+  return lim;
+}
+
 template <int D, int MT, int WK, int GEN>
 cudaError_t launch_t(const CUtensorMap* maps, const AttnParams& p, int S, int B, int Hkv,
                      cudaStream_t stream) {
   using LY = Layout<D, MT, WK>;
   const size_t smem = LY::total((p.R + 15) & ~15) + 1024;
-  // The dynamic shared-memory limit only grows (to what the largest launch
-  // so far needs), so graphs captured earlier stay launchable.
-  static size_t configured[64] = {0};
-  static bool cluster_ok[64] = {false};
-  int dev = 0;
-  cudaGetDevice(&dev);
   auto kern = verify_attn_kernel<D, MT, WK, GEN>;
-  if (dev < 64 && configured[dev] < smem) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    configured[dev] = smem;
-  }
-  if (dev < 64 && !cluster_ok[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (e != cudaSuccess) return e;
-    cluster_ok[dev] = true;
-  }
+  const cudaError_t e = ensure_kernel_limits((const void*)kern, attn_limits<D, MT, WK, GEN>(), smem, true);
+  if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(S, Hkv * p.RG, B);
   cfg.blockDim = dim3(MT * WK * 32 + 64, 1, 1);
@@ -626,17 +619,15 @@ template <int D, int MT, int WK>
 int max_cluster_t(int S, int Hkv, int B, int kbr) {
   using LY = Layout<D, MT, WK>;
   // every block path has the same shared-memory layout for a block size, and
-  // the paths used with a block size the same register budget
-  auto kern = kbr > 32 ? verify_attn_kernel<D, MT, WK, (MT >= 4 ? 2 : 1)>
-                       : verify_attn_kernel<D, MT, WK, 0>;
-  // the occupancy query needs the limit at least at the queried size; it
-  // never lowers a limit a launch has raised
-  int cur = 0;
-  cudaFuncAttributes fa;
-  if (cudaFuncGetAttributes(&fa, kern) == cudaSuccess) cur = fa.maxDynamicSharedSizeBytes;
-  if (cur < (int)(LY::total(kbr) + 1024))
-    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(LY::total(kbr) + 1024));
-  cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  // the paths used with a block size the same register budget; the occupancy
+  // query needs the limit at least at the queried size
+  constexpr int GW = MT >= 4 ? 2 : 1;
+  auto kern = kbr > 32 ? verify_attn_kernel<D, MT, WK, GW> : verify_attn_kernel<D, MT, WK, 0>;
+  KernelLimits& lim = kbr > 32 ? attn_limits<D, MT, WK, GW>() : attn_limits<D, MT, WK, 0>();
+  if (ensure_kernel_limits((const void*)kern, lim, LY::total(kbr) + 1024, true) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(S, Hkv, B);
   cfg.blockDim = dim3(MT * WK * 32 + 64, 1, 1);

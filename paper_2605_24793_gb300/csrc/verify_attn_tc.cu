@@ -779,21 +779,20 @@ size_t tc_smem_bytes() {
   return (size_t)TcLayout<D, NT>::TOTAL + 1024;
 }
 
+// Limits already set on each instantiation of the kernel.
+template <int D, int NT>
+KernelLimits& tc_limits() {
+  static KernelLimits lim;
+  return lim;
+}
+
 template <int D, int NT>
 cudaError_t launch_tc_t(const CUtensorMap* maps, const TcParams& p, int S, int B, int Hkv, int RG,
                         cudaStream_t stream) {
   const size_t smem = tc_smem_bytes<D, NT>();
-  static bool configured[64] = {false};
-  int dev = 0;
-  cudaGetDevice(&dev);
   auto kern = verify_attn_tc_kernel<D, NT>;
-  if (dev < 64 && !configured[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (e != cudaSuccess) return e;
-    configured[dev] = true;
-  }
+  const cudaError_t e = ensure_kernel_limits((const void*)kern, tc_limits<D, NT>(), smem, true);
+  if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(S, Hkv * RG, B);
   cfg.blockDim = dim3(TC_THREADS, 1, 1);
@@ -815,8 +814,10 @@ template <int D, int NT>
 int max_cluster_tc_t(int S, int Hkv, int B, int RG) {
   const size_t smem = tc_smem_bytes<D, NT>();
   auto kern = verify_attn_tc_kernel<D, NT>;
-  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (ensure_kernel_limits((const void*)kern, tc_limits<D, NT>(), smem, true) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(S, Hkv * RG, B);
   cfg.blockDim = dim3(TC_THREADS, 1, 1);

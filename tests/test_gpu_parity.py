@@ -211,6 +211,47 @@ def test_verify_attention_constant_values():
     assert torch.all(out.float() == 0.375)
 
 
+def test_verify_attention_concurrent_host_threads():
+    # Calls from several host threads (ctypes releases the GIL), each on its
+    # own stream and with its own block size, so that first launches race to
+    # set each variant's shared-memory limit: every result equals the same
+    # call made alone.
+    import threading
+    rng = np.random.default_rng(11)
+    shapes = [(2, 4, 32, 8, 128, [900, 40]), (1, 20, 32, 8, 128, [1500]),
+              (2, 40, 16, 8, 128, [300, 700]), (3, 8, 64, 8, 128, [100, 2000, 5])]
+    cases = [_paged_case(rng, *sh, True) for sh in shapes]
+    refs = []
+    for sh, t in zip(shapes, cases):
+        out = torch.empty_like(t["q"])
+        C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
+                      t["ctx_len"], out, max(sh[5]))
+        refs.append(out)
+    torch.cuda.synchronize()
+    outs = [torch.empty_like(t["q"]) for t in cases]
+    errors = []
+
+    def worker(i):
+        try:
+            s = torch.cuda.Stream()
+            t = cases[i]
+            for _ in range(20):
+                C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
+                              t["ctx_len"], outs[i], max(shapes[i][5]), stream=s)
+            s.synchronize()
+        except Exception as e:  # noqa: BLE001 - reported below
+            errors.append(e)
+
+    threads = [threading.Thread(target=worker, args=(i,)) for i in range(len(cases))]
+    for th in threads:
+        th.start()
+    for th in threads:
+        th.join()
+    assert not errors, errors
+    for ref, out in zip(refs, outs):
+        assert torch.equal(ref, out)
+
+
 LM_CASES = [
     # M, d, V, weight std
     (1, 64, 128, 0.1),
