@@ -26,6 +26,11 @@
  *    the vocabulary, a pipeline wait that timed out) skip the offending unit
  *    and set a bit in a device error word (COSPEC_DEVERR_*), which
  *    cospec_get_device_error reads and clears.  No kernel traps.
+ *  - Calls may come from any host thread and several threads at once; each
+ *    works on the calling thread's current device (its primary context is
+ *    made current on the thread's first call).  Calls that share a device
+ *    error word or the no-allocation LM-head scratch on one device see each
+ *    other's contents there.
  *  - Block geometry: a round verifies R = K + 1 rows per sequence.  Row 0 is
  *    the last token emitted by the previous round (its KV is not committed
  *    yet), rows 1..K are the draft tokens y_hat_1..y_hat_K.  Row j sits at
