@@ -670,13 +670,13 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
   const int G = Hq / Hkv;
   const int jb = G <= 64 ? 64 / G : 1;
   const int jbq = R < jb ? R : jb;
-  // More than 32 query rows per group and at least one (sequence, head, row
-  // group) per SM: the mma.sync kernel is bound by its legacy tensor-core
-  // rate there, and the tcgen05 kernel (one CTA per SM, deep ring) takes
-  // over.  Small batches stay latency-bound and keep the mma.sync kernel.
-  const long long units_g = (long long)B * Hkv * ((R + jb - 1) / jb);
+  // More than 32 query rows per group: the mma.sync kernel is bound by its
+  // legacy tensor-core rate there and the tcgen05 kernel (one CTA per SM,
+  // deep ring) takes over at every batch size (measured at batch 1, K = 15
+  // and 25, and batch 16, K = 11 and 15, on the Qwen3-8B shape).  Up to 32
+  // rows the mma.sync kernel keeps the latency-bound small batches.
   int S = 1;
-  if (tc_attn_supported(D, G) && G * jbq > 32 && units_g >= num_sms) {
+  if (tc_attn_supported(D, G) && G * jbq > 32) {
     // tcgen05 kernel: row groups of whole block rows, at most 64 query rows
     pl.kind = 1;
     pl.jb = jb;
@@ -686,15 +686,20 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
     // 128-key tiles; one CTA per SM (a stage ring of 96-192 KB); about three
     // waves of CTAs or more (finer work balances the tail: measured on the
     // Qwen3-32B batch-32 and Qwen3-8B batch-16 K = 25 workloads, 256 units
-    // ran best with 2 splits, ahead of 1 and 4), at least two tiles per CTA,
-    // no CTA with more than 64 tiles (long sequences split, so that uneven
-    // contexts balance over the waves).
+    // ran best with 2 splits, ahead of 1 and 4), at least eight tiles per
+    // CTA unless the batch is small (the prologue, the query load and the
+    // merge are fixed costs), no CTA with more than 64 tiles (long sequences
+    // split, so that uneven contexts balance over the waves).
     const int tiles_tc = (max_ctx + 127) / 128;
     pl.units = (long long)B * Hkv * pl.rg;
     const long long wave_tc = (3LL * num_sms + pl.units - 1) / (pl.units > 0 ? pl.units : 1);
     const long long len_tc = (tiles_tc + 63) / 64;
     const long long want_tc = wave_tc > len_tc ? wave_tc : len_tc;
-    while (S < 16 && S < want_tc && (S * 2) * 2 <= tiles_tc) S *= 2;
+    // a small batch (latency-bound): every cluster resident at once, and
+    // down to two tiles per CTA
+    pl.one_wave = (pl.units * 4 <= num_sms && len_tc <= 1) ? 1 : 0;
+    const int min_tiles = pl.one_wave ? 2 : 8;
+    while (S < 16 && S < want_tc && (S * 2) * min_tiles <= tiles_tc) S *= 2;
   } else {
     // Split each (sequence, head, row group) over a cluster of S CTAs: about
     // one wave of CTAs (as many as are resident at once), no CTA with more

@@ -66,7 +66,18 @@ ATTN_CASES = [
     (5, 4, 32, 8, 128, [8191, 40, 63, 64, 2049], True),
     (1, 26, 32, 8, 128, [4096], False),             # K = 25 (the paper's default): 104 rows, 2 groups
     (2, 32, 128, 8, 64, [300, 1500], True),         # 512 rows per KV head: 8 row groups
+    (2, 2, 128, 1, 128, [500, 1200], True),         # G = 128 (one KV head): 256 rows, mma.sync
 ]
+
+
+def expected_kernel(R, Hq, Hkv, D):
+    """More than 32 query rows per row group (G <= 64, head_dim 64 or 128):
+    the tcgen05 kernel; otherwise the mma.sync kernel."""
+    G = Hq // Hkv
+    if G > 64 or D not in (64, 128):
+        return C.ATTN_MMA_SYNC
+    jb = 64 // G
+    return C.ATTN_TCGEN05 if G * min(R, jb) > 32 else C.ATTN_MMA_SYNC
 
 # Batches with a (sequence, KV head, row group) per SM and more than 32 query
 # rows per group select the tcgen05 kernel.
@@ -86,7 +97,8 @@ def test_verify_attention_matches_oracle(case):
     rng = np.random.default_rng(B * 1000 + R * 100 + Hq + D + sum(ctx))
     t = _paged_case(rng, B, R, Hq, Hkv, D, ctx, shuffled)
     max_ctx = max(ctx)
-    assert C.verify_attn_plan(t["q"], t["k_pages"], t["page_table"], max_ctx)[0] == C.ATTN_MMA_SYNC
+    assert C.verify_attn_plan(t["q"], t["k_pages"], t["page_table"], max_ctx)[0] == \
+        expected_kernel(R, Hq, Hkv, D)
     out = torch.empty_like(t["q"])
     C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
                   t["ctx_len"], out, max_ctx)
@@ -106,9 +118,6 @@ def test_verify_attention_tcgen05_matches_oracle(case):
     rng = np.random.default_rng(B * 1000 + R * 100 + Hq + D + int(sum(ctx)))
     t = _paged_case(rng, B, R, Hq, Hkv, D, ctx, shuffled)
     max_ctx = int(max(ctx))
-    jb = 64 // (Hq // Hkv)
-    if C.num_sms() > B * Hkv * (-(-R // jb)):
-        pytest.skip("more SMs than (sequence, head, row group) units on this device")
     assert C.verify_attn_plan(t["q"], t["k_pages"], t["page_table"], max_ctx)[0] == C.ATTN_TCGEN05
     out = torch.empty_like(t["q"])
     C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
@@ -139,9 +148,6 @@ def test_verify_attention_tcgen05_split_matches_oracle(case):
     rng = np.random.default_rng(B * 1000 + R * 100 + Hq + D + int(sum(ctx)))
     t = _paged_case(rng, B, R, Hq, Hkv, D, ctx, shuffled)
     max_ctx = int(max(ctx))
-    jb = 64 // (Hq // Hkv)
-    if C.num_sms() > B * Hkv * (-(-R // jb)):
-        pytest.skip("more SMs than (sequence, head, row group) units on this device")
     assert C.verify_attn_plan(t["q"], t["k_pages"], t["page_table"], max_ctx) == (C.ATTN_TCGEN05, splits)
     out = torch.empty_like(t["q"])
     C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
@@ -155,8 +161,9 @@ def test_verify_attention_tcgen05_split_matches_oracle(case):
 # the whole block; K = 7 gives 17 rows, K = 25 (the paper's default) 53.
 ATTN_FULL_CASES = [
     # B, R, Hq, Hkv, D, contexts, shuffled, expected kernel
-    (1, 17, 32, 8, 128, [4096], False, 0),          # K = 7 region on a Qwen3-4B-like arbitrator
-    (3, 53, 32, 8, 128, [0, 300, 2500], True, 0),   # K = 25 region: 53 rows, 4 block-key groups of 16
+    (1, 17, 32, 8, 128, [4096], False, 1),          # K = 7 region on a Qwen3-4B-like arbitrator
+    (3, 53, 32, 8, 128, [0, 300, 2500], True, 1),   # K = 25 region: 53 rows, 4 block-key groups of 16
+    (2, 4, 128, 1, 128, [700, 90], True, 0),        # G = 128: 512 rows in 64-row groups, mma.sync
     (2, 9, 16, 8, 64, [100, 33], True, 0),          # head_dim 64, K = 3 region
     (20, 53, 8, 8, 128, _ctx(20, 6), True, 1),      # G = 1, 53 rows per group: tcgen05 kernel
     (24, 17, 32, 8, 128, _ctx(24, 7), True, 1),     # G = 4, 64-row groups: tcgen05 kernel
@@ -169,9 +176,6 @@ def test_verify_attention_full_block_matches_oracle(case):
     rng = np.random.default_rng(B * 1000 + R * 100 + Hq + D + int(sum(ctx)) + 77)
     t = _paged_case(rng, B, R, Hq, Hkv, D, ctx, shuffled)
     max_ctx = int(max(ctx))
-    jb = 64 // (Hq // Hkv)
-    if kernel == 1 and C.num_sms() > B * Hkv * (-(-R // jb)):
-        pytest.skip("more SMs than (sequence, head, row group) units on this device")
     assert C.verify_attn_plan(t["q"], t["k_pages"], t["page_table"], max_ctx)[0] == kernel
     out = torch.empty_like(t["q"])
     C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
