@@ -6,9 +6,11 @@
 // per tile) and the verify rows are N (padded to a multiple of 16, <= 256 per
 // pass), so a handful of rows still fills the tensor core and W -- the only
 // large operand -- is streamed from HBM exactly once.  Persistent CTAs (one
-// per SM) walk vocabulary tiles; warp 0 issues TMA loads (128B swizzle, W
-// with evict-first, hidden rows with evict-last) into a ring of stages,
-// warp 1 issues tcgen05.mma into one of two TMEM accumulators, warps 2-9 read
+// per SM) walk vocabulary tiles; warp 0 issues the TMA loads of W (128B
+// swizzle, evict-first) and warp 10 those of the hidden rows (evict-last) into
+// a ring of stages (one warp's bulk copies are processed one after another,
+// so two warps keep the ring full when the hidden rows are a large share of
+// each stage), warp 1 issues tcgen05.mma into one of two TMEM accumulators, warps 2-9 read
 // the finished accumulator with tcgen05.ld and fold it into per-row running
 // statistics while the next tile is multiplied.  A warp may only read the
 // TMEM lane quarter (warp id mod 4), so two epilogue warps share each quarter
@@ -31,9 +33,9 @@
 #include <cuda.h>
 #include <math.h>
 
-#include "../../include/cospec.h"
 #include <atomic>
 
+#include "../../include/cospec.h"
 #include "cospec_device.cuh"
 #include "cospec_internal.h"
 
@@ -46,7 +48,8 @@ constexpr int BK = 64;                  // K elements per stage (one 128-byte sw
 constexpr int A_BYTES = BM * BK * 2;    // 16 KB
 constexpr int EPI_WARPS = 8;            // two per TMEM lane quarter
 constexpr int EPI_THREADS = 32 * EPI_WARPS;
-constexpr int NUM_THREADS = 64 + EPI_THREADS;   // TMA warp, MMA warp, epilogue warps
+constexpr int H_WARP = 2 + EPI_WARPS;   // producer of the hidden-row boxes
+constexpr int NUM_THREADS = 64 + EPI_THREADS + 32;   // W producer, MMA, epilogue, hidden producer
 constexpr int MAX_ROWS = 256;           // rows per pass
 constexpr uint64_t WAIT_NS = 2000000000ull;
 
@@ -259,7 +262,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
   if (tid == 0) {
     for (int s = 0; s < p.stages; ++s) {
-      mbar_init(&full[s], 1);
+      mbar_init(&full[s], 2);               // the W and the hidden-row producer
       mbar_init(&empty[s], 1);
     }
     mbar_init(&tfull[0], 1);
@@ -280,11 +283,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
-  // The hidden rows may come from the previous kernel (the producer waits
-  // for it after streaming its first W stages, which do not).
+  // The hidden rows may come from the previous kernel; the W producer
+  // (warp 0) reads nothing that does and starts streaming at once.
   if (warp != 0) griddep_wait();
   uint32_t seed_lo = 0, seed_hi = 0;
-  if (warp >= 2) {
+  if (warp >= 2 && warp < H_WARP) {      // epilogue warps
     if (KEYED) {
       const unsigned long long sd = *p.seed;
       seed_lo = (uint32_t)sd;
@@ -301,28 +304,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const uint32_t idesc = idesc_bf16_f32(BM, p.n_mma);
 
   if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
+    // ------------------------------------------------------------ W producer
     if (lane == 0) {
       const uint64_t pol_w = l2_policy_evict_first();
-      const uint64_t pol_h = l2_policy_evict_last();
       int stage = 0;
       uint32_t phase = 0;
       uint32_t issued_mask = 0, issued_parity = 0;   // last load per stage (stages <= 16)
       bool ok = true;
-      // The first ring's worth of W stages streams before the wait for the
-      // previous kernel; their hidden-row boxes follow it.
+      // A warp's bulk copies are processed one after another, so the W boxes
+      // (this warp) and the hidden-row boxes (warp H_WARP) come from two
+      // warps, each arriving on the stage barrier with its own bytes.  The
+      // first ring's worth of W stages streams before the wait for the
+      // previous kernel (W does not depend on it).
       const int my_tiles = blockIdx.x < p.num_tiles ? (p.num_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
       const int npre = min(p.stages, my_tiles * kblocks);
       for (int i = 0; i < npre; ++i) {
         const int tile = blockIdx.x + (i / kblocks) * gridDim.x, kb = i % kblocks;
-        mbar_arrive_expect_tx(&full[i], (uint32_t)A_BYTES + b_bytes);
+        mbar_arrive_expect_tx(&full[i], (uint32_t)A_BYTES);
         tma_load_2d(smem_u32(smem + L.a_off + (uint32_t)i * A_BYTES), &tmap_w, &full[i], kb * BK,
                     tile * BM, pol_w);
       }
-      griddep_wait();
-      for (int i = 0; i < npre; ++i)
-        tma_load_2d(smem_u32(smem + L.b_off + (uint32_t)i * b_bytes), &tmap_h, &full[i],
-                    (i % kblocks) * BK, p.row0, pol_h);
       int li = 0;                        // loads so far, in (tile, k-block) order
       for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
         for (int kb = 0; kb < kblocks; ++kb, ++li) {
@@ -332,10 +333,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
               break;
             }
             const uint32_t sa = smem_u32(smem + L.a_off + (uint32_t)stage * A_BYTES);
-            const uint32_t sb = smem_u32(smem + L.b_off + (uint32_t)stage * b_bytes);
-            mbar_arrive_expect_tx(&full[stage], (uint32_t)A_BYTES + b_bytes);
+            mbar_arrive_expect_tx(&full[stage], (uint32_t)A_BYTES);
             tma_load_2d(sa, &tmap_w, &full[stage], kb * BK, tile * BM, pol_w);
-            tma_load_2d(sb, &tmap_h, &full[stage], kb * BK, p.row0, pol_h);
           }
           issued_mask |= 1u << stage;
           issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
@@ -349,6 +348,40 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         set_err(p.err, ERR_TIMEOUT);
         *abort_flag = 1;
         // let every issued copy land before shared memory is released
+        for (int s = 0; s < p.stages; ++s)
+          if (issued_mask & (1u << s)) mbar_wait(&full[s], (issued_parity >> s) & 1u, WAIT_NS);
+      }
+    }
+  } else if (warp == H_WARP) {
+    // ------------------------------------------------------------ hidden-row producer
+    // (after the wait on the previous kernel: the hidden rows may come from it)
+    if (lane == 0) {
+      const uint64_t pol_h = l2_policy_evict_last();
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued_mask = 0, issued_parity = 0;
+      bool ok = true;
+      int li = 0;
+      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
+        for (int kb = 0; kb < kblocks; ++kb, ++li) {
+          if (li >= p.stages && (!mbar_wait(&empty[stage], phase ^ 1u, WAIT_NS) || *abort_flag)) {
+            ok = false;
+            break;
+          }
+          const uint32_t sb = smem_u32(smem + L.b_off + (uint32_t)stage * b_bytes);
+          mbar_arrive_expect_tx(&full[stage], b_bytes);
+          tma_load_2d(sb, &tmap_h, &full[stage], kb * BK, p.row0, pol_h);
+          issued_mask |= 1u << stage;
+          issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
+          if (++stage == p.stages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        set_err(p.err, ERR_TIMEOUT);
+        *abort_flag = 1;
         for (int s = 0; s < p.stages; ++s)
           if (issued_mask & (1u << s)) mbar_wait(&full[s], (issued_parity >> s) & 1u, WAIT_NS);
       }
