@@ -511,6 +511,7 @@ def main():
 TRAFFIC = {
     ("qwen3_8b_b1", "verify_attn"): 16917504.0,
     ("qwen3_8b_b1", "lmhead_argmax_features"): 1248011008.0,
+    ("qwen3_8b_b16", "verify_attn"): 304182272.0,
     ("qwen3_32b_b32", "verify_attn"): 1362588416.0,
 }
 
