@@ -1,19 +1,22 @@
 // Verify attention of the K+1 block rows over a paged bf16 KV cache
 // (teacher-forced verification pass, Sec. 3.1 Eq. 2 of the paper).
 //
-// One CTA owns (sequence b, KV head, KV split).  The KV range of a (b, head)
-// is split over the CTAs of one thread-block cluster; every CTA streams its
-// 64-token K/V tiles (4 pages) once with TMA tensor loads -- one 3-D box per
-// page and tensor brings both 128-byte halves of the page's 16 rows,
-// 128B-swizzled, into a 3-stage mbarrier ring, the boxes of a tile issued
-// from several lanes of a producer warp at once -- and multiplies each tile against ALL query rows
-// that read this KV head (the G = Hq/Hkv heads of the group times the R block
-// rows, row index j*G + g).  Q.K^T and P.V run on bf16 tensor cores
-// (mma.m16n8k16, fp32 accumulation), the softmax is online in base 2.  The
-// block's own keys (causal inside the block) ride the same ring as a final
-// tile of the last CTA of the cluster.  Partial (max, sum, O) of the cluster
-// merge through distributed shared memory, each CTA finishing a slice of the
-// rows, so no workspace and no extra launch are needed.
+// One CTA owns (sequence b, KV head, row group of <= 64 query rows, KV
+// split).  The KV range of a (b, head) is split over the CTAs of one
+// thread-block cluster; every CTA streams its 64-token K/V tiles (4 pages)
+// once with TMA tensor loads -- one 3-D box per page and tensor brings both
+// 128-byte halves of the page's 16 rows, 128B-swizzled, into a 3-stage
+// mbarrier ring; one producer warp issues the K boxes and another the V
+// boxes (a warp's bulk copies are processed one after another) -- and
+// multiplies each tile against ALL query rows of the group that read this
+// KV head (the G = Hq/Hkv heads times the block rows, row index j*G + g).
+// Q.K^T and P.V run on bf16 tensor cores (mma.m16n8k16, fp32 accumulation),
+// the softmax is online in base 2.  The block's own keys (causal inside the
+// block, or all of them with the full mask) land in a region of their own
+// and are taken after the cache tiles by the last CTA of the cluster.
+// Partial (max, sum, O) of the cluster merge through distributed shared
+// memory, each CTA finishing a slice of the rows, so no workspace and no
+// extra launch are needed.
 #include <cuda.h>
 #include <math.h>
 
