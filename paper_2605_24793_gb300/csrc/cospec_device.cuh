@@ -278,4 +278,38 @@ CS_DEV void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
+// The sequence whose context is the `z`-th longest (ties to the lower index):
+// warp 0 ranks every sequence against all others and publishes the answer
+// through `slot` (any shared word nobody writes yet); every thread of the
+// block must call it.
+CS_DEV int sequence_by_rank(const int32_t* ctx_len, int B, int z, volatile int* slot) {
+  if ((threadIdx.x >> 5) == 0) {
+    const int lane = threadIdx.x & 31;
+    int pick = z;
+    for (int base = 0; base < B; base += 32) {
+      const int i = base + lane;
+      int r = -1;
+      if (i < B) {
+        const int ci = ctx_len[i];
+        r = 0;
+        for (int j = 0; j < B; ++j) {
+          const int cj = ctx_len[j];
+          r += (cj > ci) | ((cj == ci) & (j < i));
+        }
+      }
+      const unsigned m = __ballot_sync(0xffffffffu, r == z);
+      if (m != 0u) {
+        pick = base + __ffs(m) - 1;
+        break;
+      }
+    }
+    if (lane == 0) *slot = pick;
+  }
+  __syncthreads();
+  const int b = *slot;
+  __syncthreads();                       // the slot may be reused afterwards
+  return b;
+}
+
+
 }  // namespace cospec

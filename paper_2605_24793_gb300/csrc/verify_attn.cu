@@ -72,10 +72,11 @@ struct Layout {
   static constexpr int blk_half(int kbr) { return kbr * ROWB; }
   static constexpr int total(int kbr) { return BLK + 2 * H * kbr * ROWB; }
   // The launch adds 1024 bytes to align the base; the 2*NSTAGE+2 barriers
-  // (full[NSTAGE], empty[NSTAGE], block, received partials) take 64 bytes of
-  // that slack, before the aligned base or after the end, whichever side has
-  // room, so that two CTAs of 32 block rows still share one SM.
-  static constexpr int NBAR_BYTES = (2 * NSTAGE + 2) * 8;
+  // (full[NSTAGE], empty[NSTAGE], block, received partials) and the index of
+  // the CTA's sequence take 80 bytes of that slack, before the aligned base
+  // or after the end, whichever side has room, so that two CTAs of 32 block
+  // rows still share one SM.
+  static constexpr int NBAR_BYTES = (2 * NSTAGE + 2) * 8 + 16;   // + the sequence slot
 };
 
 // Shared-memory byte offset of 16-byte chunk `ch` (of D/8) of key row `key`
@@ -213,11 +214,12 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 64,
   uint64_t* empty = full + NSTAGE;
   uint64_t* blk_full = empty + NSTAGE;
   uint64_t* recv_bar = blk_full + 1;     // partials received from the cluster
+  volatile int* seq_slot = reinterpret_cast<volatile int*>(recv_bar + 1);   // this CTA's sequence
   uint8_t* blk_k = smem + LY::BLK;       // block keys: 2*H halves of KBR rows
 
   const int S = (int)cluster_nctarank();
   const int rank = (int)cluster_ctarank();
-  const int kvh = blockIdx.y / p.RG, rg = blockIdx.y % p.RG, b = blockIdx.z;
+  const int kvh = blockIdx.y / p.RG, rg = blockIdx.y % p.RG;
   const int row_g0 = rg * 64;                      // first query row of this group
   const int NR = min(64, p.NRT - row_g0);          // rows of this group (<= NRP)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -241,6 +243,11 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 64,
   // the wait) may come from that kernel, so the cache stream starts now.
   if (!p.kv_stable) griddep_wait();
 
+  // Sequences are taken longest context first (blockIdx.z = rank, ties by
+  // index), so that the long ones start early and the short ones fill in
+  // behind them at the end of the launch.
+  const int b = p.B > 1 ? sequence_by_rank(p.ctx_len, p.B, (int)blockIdx.z, seq_slot)
+                        : (int)blockIdx.z;
   const int C = p.ctx_len[b];
   const bool bad = (C < 0) || (C > p.max_pages * PAGE);
   if (bad && rank == 0 && kvh == 0 && tid == 0) set_err(p.err, ERR_CTX);
@@ -576,7 +583,9 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 64,
       acc.w += v.w * w;
     }
     const int j = (row_g0 + r) / p.G, g = (row_g0 + r) % p.G;
-    __nv_bfloat16* dst = p.out + (((size_t)b * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D + c;
+    // the sequence index is read again here rather than kept through the loop
+    const int bo = p.B > 1 ? *seq_slot : (int)blockIdx.z;
+    __nv_bfloat16* dst = p.out + (((size_t)bo * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D + c;
     uint2 pk;
     pk.x = pack_bf16(acc.x, acc.y);
     pk.y = pack_bf16(acc.z, acc.w);

@@ -217,7 +217,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 
   const int S = (int)cluster_nctarank();
   const int rank = (int)cluster_ctarank();
-  const int kvh = blockIdx.y / p.RG, rg = blockIdx.y % p.RG, b = blockIdx.z;
+  const int kvh = blockIdx.y / p.RG, rg = blockIdx.y % p.RG;
   const int j0 = rg * p.JB;                          // first block row of this group
   const int nj = min(p.JB, p.R - j0);
   const int NR = nj * p.G;                           // query rows of this group (<= NT)
@@ -268,6 +268,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   griddep_launch_dependents();
   if (!p.kv_stable) griddep_wait();
 
+  // Sequences are taken longest context first (blockIdx.z = rank, ties by
+  // index), so that the long ones start early and the short ones fill in
+  // behind them at the end of the launch.
+  const int b = p.B > 1 ? sequence_by_rank(p.ctx_len, p.B, (int)blockIdx.z,
+                                           reinterpret_cast<volatile int*>(red))
+                        : (int)blockIdx.z;
   const int C = p.ctx_len[b];
   const bool bad = (C < 0) || (C > p.max_pages * TPAGE);
   if (bad && rank == 0 && kvh == 0 && rg == 0 && tid == 0) set_err(p.err, ERR_CTX);
