@@ -695,17 +695,17 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
     pl.jbq = jbq;
     pl.rg = (R + pl.jb - 1) / pl.jb;
     pl.nt = ((G * pl.jbq + 15) / 16 * 16) <= 32 ? 32 : 64;
-    // 128-key tiles; one CTA per SM (a stage ring of 96-192 KB); about three
-    // waves of CTAs or more (finer work balances the tail: measured on the
-    // Qwen3-32B batch-32 and Qwen3-8B batch-16 K = 25 workloads, 256 units
-    // ran best with 2 splits, ahead of 1 and 4), at least eight tiles per
-    // CTA unless the batch is small (the prologue, the query load and the
-    // merge are fixed costs), no CTA with more than 64 tiles (long sequences
-    // split, so that uneven contexts balance over the waves).
+    // 128-key tiles; one CTA per SM (a stage ring of 96-192 KB); about one
+    // wave of CTAs or a little more (with the longest contexts started first
+    // the tail balances itself and every further split only adds merges:
+    // Qwen3-32B batch 32 ran 238 us unsplit against 255 with 2 splits,
+    // Qwen3-8B batch 16 K = 15 65 us with 2 against 87 with 4), at least
+    // eight tiles per CTA unless the batch is small (the prologue, the query
+    // load and the merge are fixed costs), no CTA with more than 256 tiles.
     const int tiles_tc = (max_ctx + 127) / 128;
     pl.units = (long long)B * Hkv * pl.rg;
-    const long long wave_tc = (3LL * num_sms + pl.units - 1) / (pl.units > 0 ? pl.units : 1);
-    const long long len_tc = (tiles_tc + 63) / 64;
+    const long long wave_tc = ((long long)num_sms + pl.units - 1) / (pl.units > 0 ? pl.units : 1);
+    const long long len_tc = (tiles_tc + 255) / 256;
     const long long want_tc = wave_tc > len_tc ? wave_tc : len_tc;
     // a small batch (latency-bound): every cluster resident at once, and
     // down to two tiles per CTA

@@ -131,14 +131,16 @@ def test_verify_attention_tcgen05_matches_oracle(case):
     assert torch.equal(out, out2)
 
 
-# Long contexts split the tcgen05 kernel's KV range over a cluster (a CTA
-# takes at most 64 tiles of 128 keys): 2, 4 and 8 splits merged through
-# distributed shared memory, with most sequences far shorter than the split.
+# The tcgen05 kernel splits a (sequence, head, row group)'s KV range over a
+# cluster when the batch has fewer units than SMs, and when a context passes
+# 256 tiles of 128 keys: 2, 4 and 8 splits merged through distributed shared
+# memory, with most sequences far shorter than the split.
 ATTN_TC_SPLIT_CASES = [
     # B, R, Hq, Hkv, D, contexts, shuffled, expected splits
-    (40, 8, 64, 8, 128, [9000] + _ctx(39, 8), True, 2),
-    (20, 16, 32, 8, 128, [20000, 3000] + _ctx(18, 9), True, 4),
-    (20, 8, 64, 8, 128, [33000, 9000] + _ctx(18, 10), False, 8),
+    (12, 8, 64, 8, 128, [6000] + _ctx(11, 8), True, 2),           # 96 units
+    (6, 8, 64, 8, 128, [9000, 3000] + _ctx(4, 9), True, 4),       # 48 units
+    (1, 8, 64, 8, 128, [6000], False, 8),                         # one wave of 8-CTA clusters
+    (20, 8, 64, 8, 128, [33000, 9000] + _ctx(18, 10), False, 2),  # a context past 256 tiles
 ]
 
 
