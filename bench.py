@@ -509,10 +509,10 @@ def main():
 # (profiles/), keyed by (workload, kernel); an entry is removed when its
 # kernel changes after the capture.
 TRAFFIC = {
-    ("qwen3_8b_b1", "verify_attn"): 16917504.0,
+    ("qwen3_8b_b1", "verify_attn"): 16918528.0,
     ("qwen3_8b_b1", "lmhead_argmax_features"): 1248011008.0,
-    ("qwen3_8b_b16", "verify_attn"): 304182272.0,
-    ("qwen3_32b_b32", "verify_attn"): 1362588416.0,
+    ("qwen3_8b_b16", "verify_attn"): 304239360.0,
+    ("qwen3_32b_b32", "verify_attn"): 1362598144.0,
 }
 
 
