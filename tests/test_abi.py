@@ -44,6 +44,8 @@ def test_status_strings(lib):
     assert lib.cospec_status_string(-1) == b"invalid argument"
     assert lib.cospec_status_string(-3) == b"workspace missing or too small"
     assert lib.cospec_status_string(123) == b"unknown status"
+    # no CUDA error recorded on this thread yet
+    assert lib.cospec_last_cuda_error() == b"cudaSuccess"
 
 
 def _dims(**kw):
