@@ -114,8 +114,9 @@ COSPEC_API int cospec_num_sms(void);
  *    CTAs of one thread-block cluster, whose partial results merge in
  *    distributed shared memory.  Two kernels implement the call: one on
  *    mma.sync tensor-core tiles, and one on tcgen05 (TMEM accumulators),
- *    used when a KV head's group has more than 32 query rows and the batch
- *    gives every SM a (sequence, KV head, row group) of its own.
+ *    used when a row group of a KV head has more than 32 query rows (and at
+ *    most 64 query heads share the KV head).  Sequences are processed
+ *    longest context first.
  *    Supported: head_dim in {64, 128}; page_size == 16; rows <= 64;
  *    num_q_heads % num_kv_heads == 0; (num_q_heads / num_kv_heads) * rows <= 512.
  * ------------------------------------------------------------------------ */
