@@ -317,6 +317,7 @@ def main():
     draft = gpu_drafts(cfg, inp)
     rnd = VerifyRound(inp, draft, cfg.lam, temperature=args.temperature,
                       seed=W.sample_seed(cfg))
+    rnd.pack_step_io()                    # one host->device and one device->host copy per step
     attn_kernel, attn_splits = C.verify_attn_plan(inp["q"][0], inp["k_pages"][0], inp["page_table"],
                                                   rnd.max_ctx)
     lm_name = "lmhead_argmax_features" if args.temperature is None else "lmhead_sample_features"
@@ -525,11 +526,12 @@ def kernels_round(k):
 
 def end_to_end(cfg, rnd, step, stream, steps, dist):
     """Per step: copy the round's activations from pinned host memory (Q and
-    the block K/V of every layer, the hidden rows, the draft ids), run the
-    round, read back the accepted lengths and emitted tokens, synchronise."""
-    srcs = [rnd.q, rnd.k_blk, rnd.v_blk, rnd.hidden, rnd.draft, rnd.draft_for_row]
+    the block K/V of every layer, the hidden rows, the draft ids; one packed
+    buffer), run the round, read back the accepted lengths and emitted tokens
+    (one packed buffer), synchronise."""
+    srcs = [rnd.io_in]
     pinned = [t.cpu().pin_memory() for t in srcs]
-    outs = [rnd.accept_len, rnd.emitted]
+    outs = [rnd.io_out]
     back = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
     h2d = sum(t.numel() * t.element_size() for t in pinned)
     d2h = sum(t.numel() * t.element_size() for t in back)

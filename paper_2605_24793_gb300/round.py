@@ -60,6 +60,33 @@ class VerifyRound:
         self.graph: Optional[torch.cuda.CUDAGraph] = None
         self.launches_per_round = self._count_launches()
 
+    def pack_step_io(self) -> None:
+        """Place the inputs a serving step receives from the host (Q and the
+        block K/V of every layer, the hidden rows, the draft ids) in one device
+        buffer ``io_in`` and the results it hands back (accepted lengths,
+        emitted tokens) in another, ``io_out``, so that a step moves each with
+        a single copy.  The tensors become views of the buffers (each slice
+        256-byte aligned); call before capturing a graph."""
+        dev = self.q.device
+        names = ("q", "k_blk", "v_blk", "hidden", "draft", "draft_for_row")
+        tensors = [getattr(self, n) for n in names]
+        sizes = [t.numel() * t.element_size() for t in tensors]
+        offs, total = [], 0
+        for n in sizes:
+            offs.append(total)
+            total += (n + 255) // 256 * 256
+        self.io_in = torch.empty(total, dtype=torch.uint8, device=dev)
+        for name, t, off, n in zip(names, tensors, offs, sizes):
+            view = self.io_in[off:off + n].view(t.dtype).view(t.shape)
+            view.copy_(t)
+            setattr(self, name, view)
+        B, R = self.cfg.batch, self.cfg.rows
+        lead = (B + 63) // 64 * 64                  # accepted lengths, then 256-byte aligned tokens
+        self.io_out = torch.zeros(lead + B * R, dtype=torch.int32, device=dev)
+        self.accept_len = self.io_out[:B]
+        self.emitted = self.io_out[lead:].view(B, R)
+        self.dims = C.attn_dims(self.q[0], self.k_pages[0], self.page_table)
+
     def _count_launches(self) -> int:
         """Kernels one round launches (attention: 1 per layer; LM head: a main
         and a merge kernel per 256-row pass; arbitration: 1 when K > 0;
