@@ -33,10 +33,13 @@ __global__ void __launch_bounds__(WARPS * 32)
   // The MLP weights do not come from the previous kernel: stage them while
   // it finishes, then wait for its statistics.
   if (mode == 0) {
-    for (int e = threadIdx.x; e < H * NF; e += blockDim.x) sm[e] = w1[e];
+    // unrolled so that several loads of a thread are in flight at once
+#pragma unroll 8
+    for (int e = threadIdx.x; e < H * NF; e += blockDim.x) sm[e] = __ldg(w1 + e);
+#pragma unroll 4
     for (int e = threadIdx.x; e < H; e += blockDim.x) {
-      sm[H * NF + e] = b1[e];
-      sm[H * NF + H + e] = w2[e];
+      sm[H * NF + e] = __ldg(b1 + e);
+      sm[H * NF + H + e] = __ldg(w2 + e);
     }
   }
   griddep_wait();
