@@ -460,6 +460,38 @@ def test_small_batched_round_with_n01_inputs():
     print(f"tie-affected sequences: {ties} of {cfg.batch}")
 
 
+def test_packed_step_buffers_give_the_same_round():
+    # The packed host-facing buffers rebind the inputs and results as views;
+    # a replayed graph over them must reproduce the unpacked round bit for bit.
+    cfg = W.CONFIGS["tiny"].replace(batch=5, ctx_lo=0, ctx_hi=900, layers=2, k=7,
+                                    shuffled_pages=True, mismatch_rate=0.5)
+    inp_ref = W.make_round_inputs(cfg, device="cuda")
+    x = O.lmhead_logits(inp_ref["hidden"].cpu(), inp_ref["w"].cpu())
+    draft = W.synth_drafts(cfg, O.topk_ids(x, 8).reshape(cfg.batch, cfg.rows, 8))
+    plain = VerifyRound(inp_ref, draft, 0.6, 0, keep_attn=True)
+    plain.replay()
+    packed = VerifyRound(W.make_round_inputs(cfg, device="cuda"), draft, 0.6, 0, keep_attn=True)
+    packed.pack_step_io()
+    assert packed.q.data_ptr() == packed.io_in.data_ptr()
+    for name in ("q", "k_blk", "v_blk", "hidden", "draft", "draft_for_row"):
+        t = getattr(packed, name)
+        assert t.data_ptr() % 256 == 0 and torch.equal(t.cpu(), getattr(plain, name).cpu())
+    packed.replay()
+    packed.replay()         # the graph restores the context: a second replay is the same round
+    torch.cuda.synchronize()
+    assert packed.accept_len.data_ptr() == packed.io_out.data_ptr()
+    for name in ("accept_len", "emitted", "argmax", "stats", "p", "accept", "ctx_len",
+                 "attn_out", "k_pages", "v_pages"):
+        a, b = getattr(plain, name).cpu(), getattr(packed, name).cpu()
+        assert torch.equal(a.view(torch.uint8) if a.is_floating_point() else a,
+                           b.view(torch.uint8) if b.is_floating_point() else b), name
+    B, R = cfg.batch, cfg.rows
+    lead = (B + 63) // 64 * 64
+    out = packed.io_out.cpu()
+    assert torch.equal(out[:B], plain.accept_len.cpu())
+    assert torch.equal(out[lead:].view(B, R), plain.emitted.cpu())
+
+
 def test_block_size_one_round_is_greedy():
     cfg, draft, ref, rnd = _tiny_round(0, 0.6, k=0, batch=3, ctx_lo=10, ctx_hi=300)
     assert np.all(rnd.accept_len.cpu().numpy() == 1)
