@@ -500,7 +500,8 @@ def main():
             "accepted_len_mean": s_mean,
             "emitted_tokens_per_s": world * cfg.batch * s_mean / (ms_per_step * 1e-3),
             "accepted_len_of": ("the one synthetic round every step replays (same drafts, "
-                                "context restored); python -m paper_2605_24793_gb300.decode measures it over many rounds"),
+                                "context restored); python -m paper_2605_24793_gb300.decode "
+                                "measures it over many rounds"),
         }
         print(json.dumps(line), flush=True)
     if dist:
