@@ -709,9 +709,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   if (S > 1) {
     cluster_wait();                      // every CTA's RECV is free and its barrier armed
     float* recv = reinterpret_cast<float*>(smem + LY::RECV);   // [S][rpo][PD] at each owner
-    if (tid == 0) {
+    // one issuing thread in each of four warps: a warp's bulk copies are
+    // processed one after another
+    if (lane == 0 && warp < 4) {
       const uint32_t recv_u = smem_u32(recv), bar_u = smem_u32(recv_bar);
-      for (int o = 0; o < S; ++o)
+      for (int o = warp; o < S; o += 4)
         bulk_copy_s2s(dsmem_map(recv_u + (uint32_t)(rank * rpo * LY::ROWP), (uint32_t)o),
                       smem_u32(part + o * rpo * PD), (uint32_t)(rpo * LY::ROWP),
                       dsmem_map(bar_u, (uint32_t)o));
@@ -744,6 +746,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     const int r = row0 + rr;
     if (r >= NR) break;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
     for (int s2 = 0; s2 < S; ++s2) {
       const float w = scl[s2 * rpo + rr];
       const float4 v = *reinterpret_cast<const float4*>(src + (s2 * rpo + rr) * PD + c);
