@@ -511,12 +511,12 @@ def main():
 
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture
 # (profiles/), keyed by (workload, kernel); an entry is removed when its
-# kernel changes after the capture.
+# kernel changes after the capture.  The attention entries (qwen3_8b_b1
+# 16918528, qwen3_8b_b16 304239360, qwen3_32b_b32 1362598144 bytes) were
+# removed when both attention kernels changed how they issue the cluster
+# merge's copies; they come back with the next capture.
 TRAFFIC = {
-    ("qwen3_8b_b1", "verify_attn"): 16918528.0,
     ("qwen3_8b_b1", "lmhead_argmax_features"): 1248011008.0,
-    ("qwen3_8b_b16", "verify_attn"): 304239360.0,
-    ("qwen3_32b_b32", "verify_attn"): 1362598144.0,
 }
 
 
