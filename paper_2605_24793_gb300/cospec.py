@@ -1,8 +1,9 @@
-"""Python binding of libcospec.so: the same four calls as include/cospec.h.
+"""Python binding of libcospec.so: the calls of include/cospec.h, same names.
 
-Argument marshalling only -- shapes are read off the tensors, pointers and
-the current CUDA stream are passed through ctypes, and every step runs in
-the library's CUDA kernels.  There is no CPU or PyTorch fallback: if the
+Argument marshalling only -- shapes are read off the tensors and checked
+against one another (a mis-shaped tensor would make a kernel read or write
+past its end), pointers and the current CUDA stream are passed through
+ctypes, and every step runs in the library's CUDA kernels.  There is no CPU or PyTorch fallback: if the
 library is missing or a call fails, an exception is raised.
 """
 from __future__ import annotations
@@ -124,6 +125,72 @@ def _req(t: torch.Tensor, dtype, name: str, ndim: Optional[int] = None):
         raise ValueError(f"{name}: expected {ndim} dims, got {t.dim()}")
 
 
+def _need(cond: bool, msg: str) -> None:
+    if not cond:
+        raise ValueError(msg)
+
+
+def _same_device(*tensors: Optional[torch.Tensor]) -> None:
+    """Every tensor on the current CUDA device (the library launches there)."""
+    dev = torch.cuda.current_device()
+    for t in tensors:
+        if t is not None and t.device.index != dev:
+            raise ValueError(f"tensor on {t.device}, but the current device is cuda:{dev}")
+
+
+def check_attn_shapes(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len, out) -> None:
+    """Shapes of one verify-attention call agree: q / out [B,R,Hq,D], block
+    K/V [B,R,Hkv,D], pools [num_pages,Hkv,P,D], page_table [B,max_pages],
+    ctx_len [B]."""
+    _need(q.dim() == 4, "q must be [B, R, Hq, D]")
+    B, R, Hq, D = q.shape
+    _need(k_pages.dim() == 4, "k_pages must be [num_pages, Hkv, P, D]")
+    _need(tuple(v_pages.shape) == tuple(k_pages.shape), "v_pages must have k_pages' shape")
+    Hkv = k_pages.shape[1]
+    _need(k_pages.shape[3] == D, "k_pages head_dim differs from q's")
+    _need(tuple(k_blk.shape) == (B, R, Hkv, D), "k_blk must be [B, R, Hkv, D]")
+    _need(tuple(v_blk.shape) == (B, R, Hkv, D), "v_blk must be [B, R, Hkv, D]")
+    _need(tuple(out.shape) == tuple(q.shape), "out must have q's shape")
+    _need(page_table.dim() == 2 and page_table.shape[0] == B, "page_table must be [B, max_pages]")
+    _need(ctx_len.dim() == 1 and ctx_len.shape[0] == B, "ctx_len must be [B]")
+
+
+def check_arbitrate_shapes(draft, argmax, stats, w1, b1, w2, mode, p_out, accept) -> None:
+    """draft [B,K]; argmax B*(K+1) ids; stats B*(K+1)*5; p_out / accept B*K;
+    for the MLP policy w1 [H,8], b1 [H], w2 [H]."""
+    _need(draft.dim() == 2, "draft must be [B, K]")
+    B, K = draft.shape
+    _need(argmax.numel() == B * (K + 1) and stats.numel() == B * (K + 1) * 5,
+          "argmax / stats must hold K+1 rows per sequence")
+    _need(p_out.numel() == B * K and accept.numel() == B * K, "p_out / accept must hold B*K values")
+    if mode == POLICY_MLP:
+        _need(w1.dim() == 2 and w1.shape[1] == 8, "w1 must be [H, 8]")
+        H = w1.shape[0]
+        _need(b1.numel() == H and w2.numel() == H, "b1 / w2 must hold H values")
+
+
+def check_commit_shapes(draft, argmax, accept, k_blk, v_blk, k_pages, v_pages, page_table,
+                        ctx_len, accept_len, emitted) -> None:
+    """draft [B,K]; argmax B*(K+1); accept B*K; block K/V [L,B,K+1,Hkv,D];
+    pools [L or 1,num_pages,Hkv,P,D]; page_table [B,max_pages]; ctx_len,
+    accept_len [B]; emitted B*(K+1)."""
+    _need(draft.dim() == 2, "draft must be [B, K]")
+    B, K = draft.shape
+    _need(argmax.numel() == B * (K + 1), "argmax must hold K+1 ids per sequence")
+    _need(accept.numel() == B * K, "accept must hold B*K values")
+    _need(k_blk.dim() == 5 and tuple(v_blk.shape) == tuple(k_blk.shape),
+          "k_blk / v_blk must both be [L, B, K+1, Hkv, D]")
+    L = k_blk.shape[0]
+    _need(k_pages.dim() == 5 and tuple(v_pages.shape) == tuple(k_pages.shape),
+          "k_pages / v_pages must both be [L, num_pages, Hkv, P, D]")
+    _need(k_pages.shape[0] in (L, 1), "pools must hold every layer, or one shared by all")
+    _need(tuple(k_blk.shape[1:]) == (B, K + 1, k_pages.shape[2], k_pages.shape[4]),
+          "k_blk must be [L, B, K+1, Hkv, D] with the pools' Hkv and D")
+    _need(page_table.dim() == 2 and page_table.shape[0] == B, "page_table must be [B, max_pages]")
+    _need(ctx_len.numel() == B and accept_len.numel() == B, "ctx_len / accept_len must be [B]")
+    _need(emitted.numel() == B * (K + 1), "emitted must hold K+1 tokens per sequence")
+
+
 def attn_dims(q: torch.Tensor, k_pages: torch.Tensor, page_table: torch.Tensor,
               softmax_scale: float = 0.0, flags: int = 0) -> AttnDims:
     """Geometry of one verify-attention call from q [B,R,Hq,D], the layer's
@@ -163,12 +230,10 @@ def verify_attn(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len, out, max
         _req(t, torch.bfloat16, n)
     _req(page_table, torch.int32, "page_table", 2)
     _req(ctx_len, torch.int32, "ctx_len", 1)
+    check_attn_shapes(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len, out)
+    _same_device(q, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len, out)
     dims = attn_dims(q, k_pages, page_table, softmax_scale,
                      (ATTN_KV_STABLE if kv_stable else 0) | (ATTN_BLOCK_FULL if block_full else 0))
-    if tuple(k_blk.shape) != (dims.batch, dims.rows, dims.num_kv_heads, dims.head_dim):
-        raise ValueError("k_blk shape does not match q / pages")
-    if out.shape != q.shape:
-        raise ValueError("out must have q's shape")
     _check(load_library().cospec_verify_attn(
         ctypes.byref(dims), int(max_ctx), _ptr(q), _ptr(k_blk), _ptr(v_blk), _ptr(k_pages),
         _ptr(v_pages), _ptr(page_table), _ptr(ctx_len), _ptr(out), _stream(stream)))
@@ -196,6 +261,7 @@ def lmhead_argmax_features(hidden, w, draft_for_row, argmax, stats, ws, stream=N
     V = w.shape[0]
     if w.shape[1] != d or draft_for_row.numel() != M or argmax.numel() != M or tuple(stats.shape) != (M, 5):
         raise ValueError("inconsistent LM-head shapes")
+    _same_device(hidden, w, draft_for_row, argmax, stats, ws)
     _check(load_library().cospec_lmhead_argmax_features(
         M, d, V, _ptr(hidden), _ptr(w), _ptr(draft_for_row), _ptr(argmax), _ptr(stats), _ptr(ws),
         ws.numel(), _stream(stream)))
@@ -221,6 +287,7 @@ def lmhead_sample_features(hidden, w, draft_for_row, temperature: float, seed, s
     V = w.shape[0]
     if w.shape[1] != d or draft_for_row.numel() != M or sample.numel() != M or tuple(stats.shape) != (M, 5):
         raise ValueError("inconsistent LM-head shapes")
+    _same_device(hidden, w, draft_for_row, seed, sample, stats, ws)
     _check(load_library().cospec_lmhead_sample_features(
         M, d, V, _ptr(hidden), _ptr(w), _ptr(draft_for_row), float(temperature), _ptr(seed),
         _ptr(sample), _ptr(stats), _ptr(ws), ws.numel(), _stream(stream)))
@@ -240,6 +307,7 @@ def lmhead_argmax_features_noalloc(hidden, w, draft_for_row, argmax, stats, stre
     V = w.shape[0]
     if w.shape[1] != d or draft_for_row.numel() != M or argmax.numel() != M or tuple(stats.shape) != (M, 5):
         raise ValueError("inconsistent LM-head shapes")
+    _same_device(hidden, w, draft_for_row, argmax, stats)
     _check(load_library().cospec_lmhead_argmax_features_noalloc(
         M, d, V, _ptr(hidden), _ptr(w), _ptr(draft_for_row), _ptr(argmax), _ptr(stats),
         _stream(stream)))
@@ -268,6 +336,7 @@ def rl_advantages(group_off, correct, round_off, match, accept, ell, params: RLP
         _req(t, torch.float32, n, 2)
         if tuple(t.shape) != (R, K):
             raise ValueError(f"{n} must be [R, K]")
+    _same_device(group_off, correct, round_off, match, accept, ell, *obj)
     dev = match.device
     out = dict(g=torch.empty((R, K), dtype=torch.float32, device=dev),
                eff=torch.empty((R, K), dtype=torch.uint8, device=dev),
@@ -299,13 +368,14 @@ def arbitrate(draft, argmax, stats, w1, b1, w2, b2: float, lam: float, mode: int
     _req(p_out, torch.float32, "p_out")
     _req(accept, torch.uint8, "accept")
     B, K = draft.shape
-    if argmax.numel() != B * (K + 1) or stats.numel() != B * (K + 1) * 5:
-        raise ValueError("argmax / stats must hold K+1 rows per sequence")
     H = 0
     if mode == POLICY_MLP:
         for t, n in ((w1, "w1"), (b1, "b1"), (w2, "w2")):
             _req(t, torch.float32, n)
         H = w1.shape[0]
+    check_arbitrate_shapes(draft, argmax, stats, w1, b1, w2, mode, p_out, accept)
+    _same_device(draft, argmax, stats, p_out, accept,
+                 *((w1, b1, w2) if mode == POLICY_MLP else ()))
     _check(load_library().cospec_arbitrate(
         B, K, _ptr(draft), _ptr(argmax), _ptr(stats), H, _ptr(w1) if mode == 0 else None,
         _ptr(b1) if mode == 0 else None, _ptr(w2) if mode == 0 else None, float(b2), float(lam),
@@ -329,11 +399,14 @@ def accept_commit(draft, argmax, accept, k_blk, v_blk, k_pages, v_pages, page_ta
     _req(ctx_len, torch.int32, "ctx_len", 1)
     _req(accept_len, torch.int32, "accept_len", 1)
     _req(emitted, torch.int32, "emitted")
+    check_commit_shapes(draft, argmax, accept, k_blk, v_blk, k_pages, v_pages, page_table,
+                        ctx_len, accept_len, emitted)
+    _same_device(draft, argmax, accept, k_blk, v_blk, k_pages, v_pages, page_table, ctx_len,
+                 accept_len, emitted)
     B, K = draft.shape
     L = k_blk.shape[0]
-    if k_pages.shape[0] not in (L, 1) or k_pages.shape != v_pages.shape or \
-            k_pages.stride(0) != v_pages.stride(0):
-        raise ValueError("k_pages / v_pages must hold the same layers with the same stride")
+    if k_pages.stride(0) != v_pages.stride(0):
+        raise ValueError("k_pages / v_pages must hold their layers with the same stride")
     # a single pool shared by every layer is passed with layer stride 0
     layer_stride = 0 if (k_pages.shape[0] == 1 and L > 1) else int(k_pages.stride(0))
     dims = AttnDims(B, K + 1, 0, k_pages.shape[2], k_pages.shape[4], k_pages.shape[3],
