@@ -194,3 +194,28 @@ def test_commit_writes_only_accepted_rows():
                 np.testing.assert_array_equal(kp2[:, pg, :, sl], kp[:, pg, :, sl])
                 np.testing.assert_array_equal(vp2[:, pg, :, sl], vp[:, pg, :, sl])
     assert touched.sum() == s.sum()
+
+
+def test_commit_hand_case_across_a_page_boundary():
+    # Page size 4.  Sequence 0 holds 3 tokens (pages 5, 2, 7 in that order)
+    # and keeps 3 block rows: positions 3, 4, 5 -> page 5 slot 3, page 2
+    # slots 0 and 1.  Sequence 1 holds 4 tokens (pages 0, 3, 1) and keeps 2:
+    # positions 4, 5 -> page 3 slots 0 and 1.  Row t of sequence b carries
+    # the value 10*b + t + 1 (K) and its negation (V); the pool starts at 0.
+    L, B, R, Hkv, D, P, num = 1, 2, 4, 1, 1, 4, 8
+    table = np.array([[5, 2, 7], [0, 3, 1]])
+    ctx = np.array([3, 4])
+    s = np.array([3, 2])
+    kb = np.zeros((L, B, R, Hkv, D), dtype=np.int16)
+    for b in range(B):
+        for t in range(R):
+            kb[0, b, t, 0, 0] = 10 * b + t + 1
+    vb = -kb
+    kp = np.zeros((L, num, Hkv, P, D), dtype=np.int16)
+    kp2, vp2, ctx2 = O.commit_kv(kb, vb, kp, kp.copy(), table, ctx, s, P)
+    expect = np.zeros((num, P), dtype=np.int16)
+    expect[5, 3], expect[2, 0], expect[2, 1] = 1, 2, 3       # sequence 0, rows 0..2
+    expect[3, 0], expect[3, 1] = 11, 12                      # sequence 1, rows 0..1
+    np.testing.assert_array_equal(kp2[0, :, 0, :, 0], expect)
+    np.testing.assert_array_equal(vp2[0, :, 0, :, 0], -expect)
+    np.testing.assert_array_equal(ctx2, [6, 6])
