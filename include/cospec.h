@@ -154,6 +154,25 @@ typedef struct {
 COSPEC_API int cospec_verify_attn_plan(const cospec_attn_dims* dims, int max_ctx, int* kernel,
                                        int* splits);
 
+/* Residency model for cospec_verify_attn_plan_model: how many clusters of
+ * `splits` CTAs of one attention kernel variant a device keeps resident at
+ * once (0: such a cluster cannot be scheduled).  kernel 0 (mma.sync):
+ * `rows` = padded query rows of a CTA (16, 32 or 64), `block_rows` = the
+ * block's keys padded to 16; kernel 1 (tcgen05): `rows` = the score tile's
+ * query columns (32 or 64), `block_rows` as for kernel 0. */
+typedef long long (*cospec_resident_fn)(int kernel, int rows, int block_rows, int splits,
+                                        void* user);
+
+/* The plan cospec_verify_attn_plan computes, for a device described by its
+ * SM count and a residency model instead of the current device (the same
+ * rules: kernel choice, KV split, one wave of resident clusters for small
+ * batches).  Host only, no CUDA call: it lets a host without a GPU check or
+ * predict the plan for any machine.  Errors as for cospec_verify_attn_plan,
+ * and COSPEC_ERR_INVALID_ARG for num_sms < 1 or a null model. */
+COSPEC_API int cospec_verify_attn_plan_model(const cospec_attn_dims* dims, int max_ctx,
+                                             int num_sms, cospec_resident_fn resident, void* user,
+                                             int* kernel, int* splits);
+
 COSPEC_API int cospec_verify_attn(const cospec_attn_dims* dims, int max_ctx,
                                   const uint16_t* q, const uint16_t* k_blk, const uint16_t* v_blk,
                                   const uint16_t* k_pages, const uint16_t* v_pages,

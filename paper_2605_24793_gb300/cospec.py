@@ -24,7 +24,7 @@ EXPORTED = ("cospec_status_string", "cospec_last_cuda_error", "cospec_get_device
             "cospec_verify_attn", "cospec_lmhead_workspace", "cospec_lmhead_argmax_features",
             "cospec_arbitrate", "cospec_accept_commit", "cospec_lmhead_argmax_features_noalloc",
             "cospec_lmhead_sample_features", "cospec_verify_attn_plan", "cospec_rl_workspace",
-            "cospec_rl_advantages")
+            "cospec_rl_advantages", "cospec_verify_attn_plan_model")
 
 
 class AttnDims(ctypes.Structure):
@@ -57,6 +57,8 @@ _lib: Optional[ctypes.CDLL] = None
 
 _vp, _i, _sz, _f = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t, ctypes.c_float
 _PDIMS = ctypes.POINTER(AttnDims)
+# cospec_resident_fn: (kernel, rows, block_rows, splits, user) -> resident clusters
+RESIDENT_FN = ctypes.CFUNCTYPE(ctypes.c_longlong, _i, _i, _i, _i, _vp)
 
 
 def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
@@ -74,6 +76,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "cospec_num_sms": (_i, []),
         "cospec_verify_attn": (_i, [_PDIMS, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
         "cospec_verify_attn_plan": (_i, [_PDIMS, _i, ctypes.POINTER(_i), ctypes.POINTER(_i)]),
+        "cospec_verify_attn_plan_model": (_i, [_PDIMS, _i, _i, RESIDENT_FN, _vp,
+                                               ctypes.POINTER(_i), ctypes.POINTER(_i)]),
         "cospec_rl_workspace": (_sz, [_i, _i]),
         "cospec_rl_advantages": (_i, [_i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp,
                                       ctypes.POINTER(RLParams), _vp, _vp, _vp, _vp, _vp, _vp, _vp,
@@ -214,6 +218,18 @@ def verify_attn_plan(q, k_pages, page_table, max_ctx: int):
     kernel, splits = ctypes.c_int(), ctypes.c_int()
     _check(load_library().cospec_verify_attn_plan(ctypes.byref(dims), int(max_ctx),
                                                   ctypes.byref(kernel), ctypes.byref(splits)))
+    return kernel.value, splits.value
+
+
+def verify_attn_plan_model(dims: AttnDims, max_ctx: int, num_sms: int, resident):
+    """(kernel, splits) of cospec_verify_attn_plan_model: the plan for a
+    device of ``num_sms`` SMs whose residency is ``resident(kernel, rows,
+    block_rows, splits)`` -> clusters resident at once.  Host only."""
+    cb = RESIDENT_FN(lambda k, r, kb, s, _user: int(resident(k, r, kb, s)))
+    kernel, splits = ctypes.c_int(), ctypes.c_int()
+    _check(load_library().cospec_verify_attn_plan_model(ctypes.byref(dims), int(max_ctx),
+                                                        int(num_sms), cb, None,
+                                                        ctypes.byref(kernel), ctypes.byref(splits)))
     return kernel.value, splits.value
 
 

@@ -233,6 +233,24 @@ COSPEC_API int cospec_verify_attn_plan(const cospec_attn_dims* d, int max_ctx, i
   return COSPEC_OK;
 }
 
+COSPEC_API int cospec_verify_attn_plan_model(const cospec_attn_dims* d, int max_ctx, int num_sms,
+                                             cospec_resident_fn resident, void* user, int* kernel,
+                                             int* splits) {
+  const int st = check_attn_dims(d);
+  if (st != COSPEC_OK) return st;
+  CS_CHECK_ARG(kernel && splits && resident && num_sms >= 1);
+  CS_CHECK_ARG(max_ctx >= 0 && max_ctx <= d->max_pages_per_seq * d->page_size);
+  const int kbr = (d->rows + 15) & ~15;
+  const AttnPlan pl = plan_verify_attn(
+      d->batch, d->rows, d->num_q_heads, d->num_kv_heads, d->head_dim, max_ctx, num_sms,
+      [=](const AttnPlan& p, int S) -> long long {
+        return resident(p.kind, p.kind == 1 ? p.nt : p.nrp, kbr, S, user);
+      });
+  *kernel = pl.kind;
+  *splits = pl.cluster;
+  return COSPEC_OK;
+}
+
 COSPEC_API int cospec_verify_attn(const cospec_attn_dims* d, int max_ctx, const uint16_t* q,
                                   const uint16_t* k_blk, const uint16_t* v_blk,
                                   const uint16_t* k_pages, const uint16_t* v_pages,

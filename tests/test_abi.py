@@ -82,6 +82,69 @@ def test_attention_plan_host_validation(lib):
     assert f(ctypes.byref(_dims()), 300 * 16 + 1, ctypes.byref(k), ctypes.byref(sp)) == -1
 
 
+# Clusters of S CTAs resident at once on a GB300 (152 SMs), from
+# cudaOccupancyMaxActiveClusters for every attention variant: two CTAs per SM
+# for the mma.sync kernel with <= 32 block keys, one otherwise (and for the
+# tcgen05 kernel).
+_GB300_TWO_PER_SM = {1: 304, 2: 152, 4: 74, 8: 36, 16: 14}
+_GB300_ONE_PER_SM = {1: 152, 2: 76, 4: 36, 8: 15, 16: 7}
+
+
+def _gb300_resident(kernel, rows, block_rows, splits):
+    table = _GB300_TWO_PER_SM if kernel == 0 and block_rows <= 32 else _GB300_ONE_PER_SM
+    return table.get(splits, 0)
+
+
+# (batch, rows, Hq, Hkv, head_dim, longest context) -> (kernel, splits): the
+# planner's choice for each workload shape, which is also the fastest of the
+# splits timed on a GB300 (Qwen3-8B batch 16: 4 splits against 2 and 8;
+# Llama-3-8B batch 64: 2 against 4 and 8; Qwen3-32B batch 32: unsplit
+# against 2; Qwen3-8B batch 16 K = 15: 2 against 4).
+PLAN_CASES = [
+    ((1, 6, 32, 8, 128, 4096), (C.ATTN_MMA_SYNC, 16)),      # Qwen3-8B, batch 1, K = 5
+    ((16, 8, 32, 8, 128, 8192), (C.ATTN_MMA_SYNC, 4)),      # Qwen3-8B, batch 16, K = 7
+    ((1, 16, 32, 8, 128, 4096), (C.ATTN_TCGEN05, 8)),       # batch 1, K = 15: one wave
+    ((16, 16, 32, 8, 128, 8192), (C.ATTN_TCGEN05, 2)),      # batch 16, K = 15
+    ((32, 8, 64, 8, 128, 16384), (C.ATTN_TCGEN05, 1)),      # Qwen3-32B, batch 32
+    ((64, 8, 32, 8, 128, 32768), (C.ATTN_MMA_SYNC, 2)),     # Llama-3-8B, batch 64
+]
+
+
+@pytest.mark.parametrize("shape,plan", PLAN_CASES, ids=lambda v: str(v))
+def test_attention_plan_on_a_gb300_model(lib, shape, plan):
+    B, R, Hq, Hkv, D, ctx = shape
+    dims = C.AttnDims(B, R, Hq, Hkv, D, 16, (ctx + R + 15) // 16, 1 << 20, 0.0, 0)
+    assert C.verify_attn_plan_model(dims, ctx, 152, _gb300_resident) == plan
+
+
+def test_attention_plan_model_rules(lib):
+    # a batch of a few units: the largest split whose clusters are all resident
+    dims = C.AttnDims(1, 6, 32, 8, 128, 16, 300, 1 << 20, 0.0, 0)
+    assert C.verify_attn_plan_model(dims, 4096, 152, lambda k, r, kb, s: 304 // s) == (0, 16)
+    assert C.verify_attn_plan_model(dims, 4096, 152, lambda k, r, kb, s: 7 if s >= 16 else 304 // s) \
+        == (0, 8)
+    # no cluster of more than one CTA can be scheduled: no split
+    assert C.verify_attn_plan_model(dims, 4096, 152, lambda k, r, kb, s: 152 if s == 1 else 0) \
+        == (0, 1)
+    # short contexts: at least four 64-key tiles per CTA (256 keys -> 1 split)
+    assert C.verify_attn_plan_model(dims, 256, 152, _gb300_resident) == (0, 1)
+    assert C.verify_attn_plan_model(dims, 512, 152, _gb300_resident) == (0, 2)
+    # more than 32 query rows per row group with G <= 64: the tcgen05 kernel;
+    # a KV head shared by 128 query heads stays on the mma.sync kernel
+    big = C.AttnDims(4, 8, 64, 8, 128, 16, 300, 1 << 20, 0.0, 0)
+    assert C.verify_attn_plan_model(big, 4096, 152, _gb300_resident)[0] == C.ATTN_TCGEN05
+    g128 = C.AttnDims(4, 2, 128, 1, 128, 16, 300, 1 << 20, 0.0, 0)
+    assert C.verify_attn_plan_model(g128, 4096, 152, _gb300_resident)[0] == C.ATTN_MMA_SYNC
+    # argument checks
+    f = lib.cospec_verify_attn_plan_model
+    k, sp = ctypes.c_int(), ctypes.c_int()
+    cb = C.RESIDENT_FN(lambda *a: 1)
+    assert f(ctypes.byref(dims), 4096, 0, cb, None, ctypes.byref(k), ctypes.byref(sp)) == -1
+    assert f(ctypes.byref(dims), 4096, 152, C.RESIDENT_FN(), None, ctypes.byref(k),
+             ctypes.byref(sp)) == -1
+    assert f(ctypes.byref(dims), 300 * 16 + 1, 152, cb, None, ctypes.byref(k), ctypes.byref(sp)) == -1
+
+
 def test_lmhead_host_validation(lib):
     f = lib.cospec_lmhead_argmax_features
     assert f(0, 4096, 1000, *([None] * 6), 0, None) == 0          # no rows: nothing to do
