@@ -88,6 +88,8 @@ ATTN_TC_CASES = [
     (10, 8, 128, 8, 128, _ctx(10, 3), True),        # 128 rows: two row groups
     (20, 8, 40, 8, 128, _ctx(20, 4), False),        # G = 5: 40 rows
     (20, 16, 32, 8, 128, [2000] + _ctx(19, 5), True),  # G = 4, 16 block rows: 64 rows, longer context
+    (3, 64, 8, 8, 128, [0, 100, 1500], True),        # R = 64, the largest block: 64 rows per group
+    (2, 64, 16, 8, 64, [50, 700], True),             # R = 64, G = 2: two 64-row groups, head_dim 64
 ]
 
 
@@ -169,6 +171,7 @@ ATTN_FULL_CASES = [
     (2, 9, 16, 8, 64, [100, 33], True, 0),          # head_dim 64, K = 3 region
     (20, 53, 8, 8, 128, _ctx(20, 6), True, 1),      # G = 1, 53 rows per group: tcgen05 kernel
     (24, 17, 32, 8, 128, _ctx(24, 7), True, 1),     # G = 4, 64-row groups: tcgen05 kernel
+    (2, 64, 8, 8, 128, [300, 0], True, 1),          # a 64-row region, the largest block
 ]
 
 
