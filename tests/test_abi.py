@@ -4,6 +4,8 @@ anything (no GPU needed)."""
 import ctypes
 import os
 import re
+import shutil
+import subprocess
 
 import pytest
 
@@ -194,3 +196,40 @@ def test_sample_host_validation(lib):
     assert f(*args(1.0, ctypes.c_void_p((1 << 20) + 4))) == -1        # seed not 8-byte aligned
     assert f(0, 4096, 1000, *([None] * 3), 1.0, None, None, None, None, 0, None) == 0
     assert f(4, 4000, 1000, fake, fake, fake, 1.0, fake, fake, fake, fake, 1 << 30, None) == -2
+
+
+C_PROGRAM = r"""
+#include <stdio.h>
+#include <string.h>
+#include "cospec.h"
+int main(void) {
+  cospec_attn_dims d;
+  int kernel = -1, splits = -1;
+  memset(&d, 0, sizeof d);
+  d.batch = 1; d.rows = 6; d.num_q_heads = 32; d.num_kv_heads = 8; d.head_dim = 96;
+  d.page_size = 16; d.max_pages_per_seq = 300; d.num_pages = 300;
+  if (strcmp(cospec_status_string(COSPEC_OK), "ok") != 0) return 1;
+  if (cospec_verify_attn_plan(&d, 4096, &kernel, &splits) != COSPEC_ERR_UNSUPPORTED) return 2;
+  if (cospec_lmhead_argmax_features(0, 4096, 1000, NULL, NULL, NULL, NULL, NULL, NULL, 0,
+                                    NULL) != COSPEC_OK) return 3;
+  puts("c abi ok");
+  return 0;
+}
+"""
+
+
+def test_header_is_plain_c_and_links(lib, tmp_path):
+    # the header compiles as strict C99 and a C program links and calls the library
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "abi.c"
+    src.write_text(C_PROGRAM)
+    exe = tmp_path / "abi"
+    libdir = os.path.dirname(C.LIB_PATH)
+    r = subprocess.run([gcc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror",
+                        "-I", os.path.join(ROOT, "include"), str(src), "-L", libdir, "-lcospec",
+                        f"-Wl,-rpath,{libdir}", "-o", str(exe)], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    out = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
+    assert out.returncode == 0 and out.stdout.strip() == "c abi ok", (out.returncode, out.stderr)
