@@ -47,3 +47,23 @@ def test_gpu_arm_fails_loudly_without_a_gpu():
     r = _run("--config", "tiny", "--steps", "2", "--warmup", "3", "--no-cpu-baseline")
     assert r.returncode != 0
     assert _json_lines(r.stdout) == []
+
+
+def _free_port():
+    import socket
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def test_reference_arm_under_torchrun_prints_once():
+    # two ranks launched the way the driver launches N > 1: rank 0 alone runs
+    # the reference arm and prints; the other rank exits 0 without a line
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+           "--master-addr", "127.0.0.1", "--master-port", str(_free_port()),
+           os.path.join(ROOT, "bench.py"), "--impl", "reference", "--config", "tiny", "--gpus", "2",
+           "--steps", "2", "--warmup", "3"]
+    r = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = _json_lines(r.stdout)
+    assert len(lines) == 1 and lines[0]["impl"] == "reference" and lines[0]["n_gpus"] == 2
