@@ -4,6 +4,7 @@ reads, and the GPU arm fails loudly, with no JSON line, when there is no
 GPU (there is no CPU fallback)."""
 import json
 import os
+import socket
 import subprocess
 import sys
 
@@ -50,7 +51,6 @@ def test_gpu_arm_fails_loudly_without_a_gpu():
 
 
 def _free_port():
-    import socket
     with socket.socket() as s:
         s.bind(("127.0.0.1", 0))
         return s.getsockname()[1]
