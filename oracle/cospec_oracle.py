@@ -28,6 +28,12 @@ Pins (what fixes each function other than itself; see tests/test_oracle_*.py):
                         Eq. 15, exhaustive comparison with the sequential
                         procedure of App. F (Inference Procedure).
   commit_kv             byte equality of touched / untouched slots.
+  cospec_round          a whole round built by hand (identity LM head, rows
+                        with two live logits, one mismatch, a three-unit MLP,
+                        a two-layer commit across a page boundary): which row
+                        scores which draft token, the bonus row's NaN, the
+                        rows each position's features read, s, the emitted
+                        tokens, key margins, per-layer pools.
 """
 from __future__ import annotations
 
