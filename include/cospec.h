@@ -64,8 +64,9 @@ typedef enum {
 
 /* Bits of the device error word. */
 #define COSPEC_DEVERR_PAGE 1     /* page id outside [0, num_pages) */
-#define COSPEC_DEVERR_CTX 2      /* ctx_len < 0, ctx_len > max_ctx (attention), or ctx_len plus the
-                                    accepted rows > max_pages_per_seq * page_size (commit) */
+#define COSPEC_DEVERR_CTX 2      /* ctx_len < 0 or ctx_len > max_pages_per_seq * page_size
+                                    (attention), or ctx_len plus the accepted rows >
+                                    max_pages_per_seq * page_size (commit) */
 #define COSPEC_DEVERR_TOKEN 4    /* token id outside the vocabulary */
 #define COSPEC_DEVERR_TIMEOUT 8  /* a bounded pipeline wait gave up (never expected) */
 #define COSPEC_DEVERR_OFFSETS 16 /* a group / round offset array is not non-decreasing within
@@ -109,7 +110,10 @@ COSPEC_API int cospec_num_sms(void);
  *             first ceil(ctx_len[b] / page_size) entries are read.
  *    ctx_len  int32 [batch]
  *    out      bf16 [batch, rows, num_q_heads, head_dim] (may not alias inputs)
- *    max_ctx  an upper bound of ctx_len[*] (host-side; sizes the KV split)
+ *    max_ctx  the expected largest ctx_len[*] (host-side; 0 <= max_ctx <=
+ *             max_pages_per_seq * page_size).  It only sizes the KV split: a
+ *             context above it is still attended in full and correctly, only
+ *             with a split planned for a shorter one; it sets no error bit.
  *    No workspace: the KV range of a (sequence, KV head) is split over the
  *    CTAs of one thread-block cluster, whose partial results merge in
  *    distributed shared memory.  Two kernels implement the call: one on
@@ -296,8 +300,11 @@ COSPEC_API int cospec_arbitrate(int B, int K, const int32_t* draft, const int32_
  *    k_blk, v_blk  bf16 [num_layers, B, K+1, num_kv_heads, head_dim]
  *    k_pages, v_pages  bf16: layer l's pool [num_pages, num_kv_heads,
  *             page_size, head_dim] starts pool_layer_stride elements after
- *             layer l-1's (pool_layer_stride >= num_pages*Hkv*P*D, or 0 when
- *             every layer shares one pool)
+ *             layer l-1's.  With num_layers > 1, pool_layer_stride must be
+ *             >= num_pages*Hkv*P*D (layers never share cells; 0 or a smaller
+ *             stride returns COSPEC_ERR_INVALID_ARG); with num_layers == 1 it
+ *             is ignored.  A pool that stands for several layers at once is
+ *             committed with num_layers = 1 and one layer's staging rows.
  *    dims     the attention geometry (batch == B, rows == K+1)
  *    ctx_len  int32 [B], updated in place
  *    accept_len int32 [B]; emitted int32 [B, K+1] (padded with -1)

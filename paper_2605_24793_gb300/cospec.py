@@ -423,8 +423,13 @@ def accept_commit(draft, argmax, accept, k_blk, v_blk, k_pages, v_pages, page_ta
     L = k_blk.shape[0]
     if k_pages.stride(0) != v_pages.stride(0):
         raise ValueError("k_pages / v_pages must hold their layers with the same stride")
-    # a single pool shared by every layer is passed with layer stride 0
-    layer_stride = 0 if (k_pages.shape[0] == 1 and L > 1) else int(k_pages.stride(0))
+    # A single pool standing for every layer receives layer 0's rows only (the
+    # library rejects several layers committed into one pool: their writes
+    # would race for the same cells).
+    if k_pages.shape[0] == 1 and L > 1:
+        L = 1
+        k_blk, v_blk = k_blk[:1], v_blk[:1]
+    layer_stride = int(k_pages.stride(0))
     dims = AttnDims(B, K + 1, 0, k_pages.shape[2], k_pages.shape[4], k_pages.shape[3],
                     page_table.shape[1], k_pages.shape[1], 0.0, 0)
     dims.num_q_heads = dims.num_kv_heads

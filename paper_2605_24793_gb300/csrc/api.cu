@@ -132,10 +132,15 @@ using namespace cospec;
 // The CUDA error behind this host thread's last COSPEC_ERR_CUDA.
 static thread_local cudaError_t t_last_cuda_error = cudaSuccess;
 
-static int from_cuda(cudaError_t e) {
+int cospec::cuda_status(cudaError_t e) {
   if (e == cudaSuccess) return COSPEC_OK;
   t_last_cuda_error = e;
   return COSPEC_ERR_CUDA;
+}
+
+int cospec::cuda_lookup_failed() {
+  const cudaError_t e = cudaPeekAtLastError();
+  return cuda_status(e == cudaSuccess ? cudaErrorUnknown : e);
 }
 
 extern "C" {
@@ -160,13 +165,13 @@ COSPEC_API int cospec_get_device_error(int* flags, void* stream) {
   CS_CHECK_ARG(flags != nullptr);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   int* dptr = device_error_word();
-  if (!dptr) return COSPEC_ERR_CUDA;
+  if (!dptr) return cuda_lookup_failed();
   int v = 0;
-  if (cudaStreamSynchronize(st) != cudaSuccess) return COSPEC_ERR_CUDA;
-  if (cudaMemcpyAsync(&v, dptr, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess)
-    return COSPEC_ERR_CUDA;
-  if (cudaMemsetAsync(dptr, 0, sizeof(int), st) != cudaSuccess) return COSPEC_ERR_CUDA;
-  if (cudaStreamSynchronize(st) != cudaSuccess) return COSPEC_ERR_CUDA;
+  cudaError_t e = cudaStreamSynchronize(st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&v, dptr, sizeof(int), cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(dptr, 0, sizeof(int), st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return cuda_status(e);
   *flags = v;
   return v ? COSPEC_ERR_DEVICE_CHECK : COSPEC_OK;
 }
@@ -226,7 +231,7 @@ COSPEC_API int cospec_verify_attn_plan(const cospec_attn_dims* d, int max_ctx, i
   CS_CHECK_ARG(kernel && splits);
   CS_CHECK_ARG(max_ctx >= 0 && max_ctx <= d->max_pages_per_seq * d->page_size);
   const int sms = device_num_sms();
-  if (sms <= 0) return COSPEC_ERR_CUDA;
+  if (sms <= 0) return cuda_lookup_failed();
   const AttnPlan pl = attn_plan(d, max_ctx, sms);
   *kernel = pl.kind;
   *splits = pl.cluster;
@@ -264,10 +269,10 @@ COSPEC_API int cospec_verify_attn(const cospec_attn_dims* d, int max_ctx, const 
   CS_CHECK_ARG(aligned16(q) && aligned16(k_blk) && aligned16(v_blk) && aligned16(k_pages) &&
                aligned16(v_pages) && aligned16(out));
   const int sms = device_num_sms();
-  if (sms <= 0) return COSPEC_ERR_CUDA;
+  if (sms <= 0) return cuda_lookup_failed();
   const AttnPlan pl = attn_plan(d, max_ctx, sms);
   int* err = device_error_word();
-  if (!err) return COSPEC_ERR_CUDA;
+  if (!err) return cuda_lookup_failed();
   AttnArgs a{};
   a.q = reinterpret_cast<const __nv_bfloat16*>(q);
   a.k_blk = reinterpret_cast<const __nv_bfloat16*>(k_blk);
@@ -289,7 +294,7 @@ COSPEC_API int cospec_verify_attn(const cospec_attn_dims* d, int max_ctx, const 
   a.max_ctx = max_ctx;
   a.kv_stable = (d->flags & COSPEC_ATTN_KV_STABLE) ? 1 : 0;
   a.block_full = (d->flags & COSPEC_ATTN_BLOCK_FULL) ? 1 : 0;
-  return from_cuda(launch_verify_attn(a, pl, err, static_cast<cudaStream_t>(stream)));
+  return cuda_status(launch_verify_attn(a, pl, err, static_cast<cudaStream_t>(stream)));
 }
 
 // ---------------------------------------------------------------- LM head
@@ -310,12 +315,12 @@ COSPEC_API int cospec_lmhead_argmax_features(int M, int d, int V, const uint16_t
   if ((long long)V > 0x7fffff00LL) return COSPEC_ERR_UNSUPPORTED;
   CS_CHECK_ARG(aligned16(hidden) && aligned16(w));
   const int sms = device_num_sms();
-  if (sms <= 0) return COSPEC_ERR_CUDA;
+  if (sms <= 0) return cuda_lookup_failed();
   const LmheadPlan pl = plan_lmhead(M, d, V, sms);
   if (!ws || ws_bytes < pl.ws_bytes || !aligned16(ws)) return COSPEC_ERR_WORKSPACE;
   int* err = device_error_word();
-  if (!err) return COSPEC_ERR_CUDA;
-  return from_cuda(launch_lmhead(M, d, V, reinterpret_cast<const __nv_bfloat16*>(hidden),
+  if (!err) return cuda_lookup_failed();
+  return cuda_status(launch_lmhead(M, d, V, reinterpret_cast<const __nv_bfloat16*>(hidden),
                                  reinterpret_cast<const __nv_bfloat16*>(w), draft_for_row, argmax,
                                  stats, ws, pl, err, static_cast<cudaStream_t>(stream)));
 }
@@ -334,12 +339,12 @@ COSPEC_API int cospec_lmhead_sample_features(int M, int d, int V, const uint16_t
   if ((long long)V > 0x7fffff00LL) return COSPEC_ERR_UNSUPPORTED;
   CS_CHECK_ARG(aligned16(hidden) && aligned16(w));
   const int sms = device_num_sms();
-  if (sms <= 0) return COSPEC_ERR_CUDA;
+  if (sms <= 0) return cuda_lookup_failed();
   const LmheadPlan pl = plan_lmhead(M, d, V, sms);
   if (!ws || ws_bytes < pl.ws_bytes || !aligned16(ws)) return COSPEC_ERR_WORKSPACE;
   int* err = device_error_word();
-  if (!err) return COSPEC_ERR_CUDA;
-  return from_cuda(launch_lmhead(M, d, V, reinterpret_cast<const __nv_bfloat16*>(hidden),
+  if (!err) return cuda_lookup_failed();
+  return cuda_status(launch_lmhead(M, d, V, reinterpret_cast<const __nv_bfloat16*>(hidden),
                                  reinterpret_cast<const __nv_bfloat16*>(w), draft_for_row, sample,
                                  stats, ws, pl, err, static_cast<cudaStream_t>(stream),
                                  reinterpret_cast<const unsigned long long*>(seed),
@@ -361,7 +366,7 @@ COSPEC_API int cospec_arbitrate(int B, int K, const int32_t* draft, const int32_
     CS_CHECK_ARG(w1 && b1 && w2 && mlp_hidden >= 1 && !isnan(b2));
     if (mlp_hidden > 1024) return COSPEC_ERR_UNSUPPORTED;
   }
-  return from_cuda(launch_arbitrate(B, K, draft, argmax, stats, mlp_hidden, w1, b1, w2, b2, lambda,
+  return cuda_status(launch_arbitrate(B, K, draft, argmax, stats, mlp_hidden, w1, b1, w2, b2, lambda,
                                     policy_mode, p_out, accept, static_cast<cudaStream_t>(stream)));
 }
 
@@ -386,11 +391,14 @@ COSPEC_API int cospec_accept_commit(int B, int K, int num_layers, const cospec_a
   if (num_layers > 0) {
     CS_CHECK_ARG(k_blk && v_blk && k_pages && v_pages);
     CS_CHECK_ARG(aligned16(k_blk) && aligned16(v_blk) && aligned16(k_pages) && aligned16(v_pages));
-    CS_CHECK_ARG(num_layers == 1 || pool_layer_stride == 0 || pool_layer_stride >= pool_elems);
+    // Several layers need pools of their own: with one pool shared by all
+    // layers, every layer's rows would land in the same cells and the
+    // committed bytes would depend on which write came last.
+    CS_CHECK_ARG(num_layers == 1 || pool_layer_stride >= pool_elems);
     CS_CHECK_ARG(pool_layer_stride % 8 == 0);
   }
   int* err = device_error_word();
-  if (!err) return COSPEC_ERR_CUDA;
+  if (!err) return cuda_lookup_failed();
   CommitArgs a{};
   a.B = B;
   a.K = K;
@@ -412,7 +420,7 @@ COSPEC_API int cospec_accept_commit(int B, int K, int num_layers, const cospec_a
   a.ctx_len = ctx_len;
   a.accept_len = accept_len;
   a.emitted = emitted;
-  return from_cuda(launch_accept_commit(a, err, static_cast<cudaStream_t>(stream)));
+  return cuda_status(launch_accept_commit(a, err, static_cast<cudaStream_t>(stream)));
 }
 
 }  // extern "C"

@@ -45,6 +45,13 @@ struct KernelLimits {
 // launchable) and, with `cluster`, allow non-portable cluster sizes.  Calls
 // from several host threads are serialised; later calls that need nothing
 // new only read `lim`.
+// Records e as the calling thread's last CUDA error (cospec_last_cuda_error)
+// and returns COSPEC_ERR_CUDA, or COSPEC_OK for cudaSuccess.
+int cuda_status(cudaError_t e);
+// The same for a failed lookup that returned no cudaError_t: records the
+// runtime's pending error (cudaErrorUnknown if there is none).
+int cuda_lookup_failed();
+
 cudaError_t ensure_kernel_limits(const void* kern, KernelLimits& lim, size_t smem_bytes,
                                  bool cluster);
 

@@ -696,15 +696,21 @@ static __device__ __align__(256) unsigned char g_lmhead_scratch[NOALLOC_ENTRIES 
 
 std::atomic<void*> g_scratch_addr[64];   // per device; a race only repeats the lookup
 
-void* scratch_address() {
+// The scratch's device address on the current device, looked up on the
+// device's first call; the CUDA error of a failed lookup otherwise.
+cudaError_t scratch_address(void** out) {
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   void* addr = g_scratch_addr[dev].load(std::memory_order_acquire);
   if (!addr) {
-    if (cudaGetSymbolAddress(&addr, g_lmhead_scratch) != cudaSuccess) return nullptr;
+    e = cudaGetSymbolAddress(&addr, g_lmhead_scratch);
+    if (e != cudaSuccess) return e;
     g_scratch_addr[dev].store(addr, std::memory_order_release);
   }
-  return addr;
+  *out = addr;
+  return cudaSuccess;
 }
 
 }  // namespace
@@ -723,22 +729,24 @@ extern "C" COSPEC_API int cospec_lmhead_argmax_features_noalloc(
     return COSPEC_ERR_INVALID_ARG;
   if (M > NOALLOC_MAX_M) return COSPEC_ERR_UNSUPPORTED;          // beyond the fixed scratch
   const int sms = device_num_sms();
-  if (sms <= 0) return COSPEC_ERR_CUDA;
+  if (sms <= 0) return cuda_lookup_failed();
   const LmheadPlan pl = plan_lmhead(M, d, V, sms);
   if (pl.grid > NOALLOC_MAX_CTAS) return COSPEC_ERR_UNSUPPORTED;  // beyond the fixed scratch
-  void* scratch = scratch_address();
+  void* scratch = nullptr;
+  const cudaError_t se = scratch_address(&scratch);
+  if (se != cudaSuccess) return cuda_status(se);
   int* err = device_error_word();
-  if (!scratch || !err) return COSPEC_ERR_CUDA;
+  if (!err) return cuda_lookup_failed();
   float4* part = static_cast<float4*>(scratch);
   int* part_idx = reinterpret_cast<int*>(part + NOALLOC_ENTRIES);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   CUtensorMap map_w, map_h;
   if (!make_map(&map_w, w, (uint64_t)V, (uint64_t)d, BM) ||
       !make_map(&map_h, hidden, (uint64_t)M, (uint64_t)d, (uint32_t)pl.n_mma))
-    return COSPEC_ERR_CUDA;
-  if (ensure_kernel_limits((const void*)lmhead_kernel<false>, lm_limits<false>(), 227 * 1024, false) !=
-      cudaSuccess)
-    return COSPEC_ERR_CUDA;
+    return cuda_status(cudaErrorInvalidValue);      // as the workspace entry point reports it
+  const cudaError_t le =
+      ensure_kernel_limits((const void*)lmhead_kernel<false>, lm_limits<false>(), 227 * 1024, false);
+  if (le != cudaSuccess) return cuda_status(le);
   uint32_t tmem_cols = 32;
   while (tmem_cols < (uint32_t)(2 * pl.n_mma)) tmem_cols <<= 1;
   // Each pass overwrites every scratch entry its merge kernel reads, so the
@@ -758,13 +766,13 @@ extern "C" COSPEC_API int cospec_lmhead_argmax_features_noalloc(
     p.stages = pl.stages;
     p.tmem_cols = tmem_cols;
     p.err = err;
-    if (launch_pdl(lmhead_kernel<false>, dim3(pl.grid), dim3(NUM_THREADS), pl.smem_bytes, st,
-                   map_w, map_h, p) != cudaSuccess)
-      return COSPEC_ERR_CUDA;
-    if (launch_pdl(lmhead_reduce_kernel<false>, dim3((p.n_rows + 3) / 4), dim3(128), 0, st,
-                   (const float4*)part, (const int*)part_idx, (const float*)nullptr, pl.grid,
-                   p.row0, p.n_rows, V, draft_for_row, argmax, stats, err) != cudaSuccess)
-      return COSPEC_ERR_CUDA;
+    cudaError_t e = launch_pdl(lmhead_kernel<false>, dim3(pl.grid), dim3(NUM_THREADS),
+                               pl.smem_bytes, st, map_w, map_h, p);
+    if (e == cudaSuccess)
+      e = launch_pdl(lmhead_reduce_kernel<false>, dim3((p.n_rows + 3) / 4), dim3(128), 0, st,
+                     (const float4*)part, (const int*)part_idx, (const float*)nullptr, pl.grid,
+                     p.row0, p.n_rows, V, draft_for_row, argmax, stats, err);
+    if (e != cudaSuccess) return cuda_status(e);
   }
   return COSPEC_OK;
 }

@@ -287,7 +287,7 @@ extern "C" COSPEC_API int cospec_rl_advantages(
   const size_t need = cospec_rl_workspace(num_groups, num_rollouts);
   if (!ws || ws_bytes < need) return COSPEC_ERR_WORKSPACE;
   int* err = device_error_word();
-  if (!err) return COSPEC_ERR_CUDA;
+  if (!err) return cuda_lookup_failed();
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(ws) + 255) & ~uintptr_t(255));
   const size_t mb = align256((size_t)num_rollouts * sizeof(double));
@@ -321,12 +321,12 @@ extern "C" COSPEC_API int cospec_rl_advantages(
   if (num_groups > 0) {
     rl_group_kernel<<<num_groups, RL_THREADS, 0, st>>>(a);
     const cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return COSPEC_ERR_CUDA;
+    if (e != cudaSuccess) return cuda_status(e);
   }
   if (have_obj) {
     rl_loss_kernel<<<1, RL_THREADS, 0, st>>>(a.part, num_groups, pr, loss);
     const cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return COSPEC_ERR_CUDA;
+    if (e != cudaSuccess) return cuda_status(e);
   }
   return COSPEC_OK;
 }

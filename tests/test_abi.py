@@ -6,8 +6,10 @@ import os
 import re
 import shutil
 import subprocess
+import threading
 
 import pytest
+import torch
 
 from paper_2605_24793_gb300 import build as B
 from paper_2605_24793_gb300 import cospec as C
@@ -159,6 +161,31 @@ def test_lmhead_host_validation(lib):
     assert lib.cospec_lmhead_workspace(6, 4096, 151936) > 0
 
 
+def test_cuda_failure_is_recorded_without_a_device(lib):
+    # On a host without a GPU every call that gets past its argument checks
+    # fails in its first CUDA call; that error is what cospec_last_cuda_error
+    # then names (per host thread: run in a fresh one).
+    if torch.cuda.is_available():
+        pytest.skip("needs a host without a GPU")
+    fake = ctypes.c_void_p(1 << 20)                                # never dereferenced
+    got = {}
+
+    def run():
+        got["before"] = lib.cospec_last_cuda_error()
+        got["status"] = lib.cospec_lmhead_argmax_features_noalloc(6, 4096, 1000, fake, fake, fake,
+                                                                  fake, fake, None)
+        got["after"] = lib.cospec_last_cuda_error()
+        got["ws"] = lib.cospec_lmhead_argmax_features(6, 4096, 1000, fake, fake, fake, fake, fake,
+                                                      fake, 1 << 30, None)
+
+    t = threading.Thread(target=run)
+    t.start()
+    t.join()
+    assert got["before"] == b"cudaSuccess"
+    assert got["status"] == -4 and got["ws"] == -4
+    assert got["after"] not in (b"cudaSuccess", b"cudaErrorUnknown")
+
+
 def test_arbitrate_host_validation(lib):
     f = lib.cospec_arbitrate
     fake = ctypes.c_void_p(1 << 20)
@@ -180,6 +207,9 @@ def test_commit_host_validation(lib):
     assert f(2, 4, 36, ctypes.byref(d), *args, 10 ** 9, fake, fake, fake, fake, None) == -1
     # layer stride smaller than one pool
     assert f(2, 5, 36, ctypes.byref(d), *args, 1024, fake, fake, fake, fake, None) == -1
+    # several layers into one shared pool (stride 0) would race for the same cells
+    assert f(2, 5, 36, ctypes.byref(d), *args, 0, fake, fake, fake, fake, None) == -1
+    assert f(2, 5, 2, ctypes.byref(d), *args, 0, fake, fake, fake, fake, None) == -1
     assert f(2, 5, 36, ctypes.byref(d), *([None] * 7), 10 ** 9, fake, fake, fake, fake, None) == -1
 
 

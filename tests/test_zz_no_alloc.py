@@ -27,9 +27,10 @@ def test_noalloc_matches_workspace_entry_point_on_consecutive_calls():
     lib = C.load_library(BLD.build())
     torch.cuda.set_device(0)
     rng = np.random.default_rng(2024)
-    # two different problems back to back: the second call must not see the
-    # first call's scratch contents
-    for M, d, V in ((6, 4096, 151936), (300, 512, 5000)):
+    # different problems back to back: a call must not see an earlier call's
+    # scratch contents; M = 512 runs two full 256-row passes that reuse the
+    # scratch inside one call
+    for M, d, V in ((6, 4096, 151936), (300, 512, 5000), (512, 1024, 40000)):
         hidden = torch.from_numpy(rng.standard_normal((M, d), dtype=np.float32)).to(torch.bfloat16).cuda()
         w = torch.from_numpy(rng.standard_normal((V, d), dtype=np.float32) * 0.05).to(torch.bfloat16).cuda()
         dfr = torch.from_numpy(rng.integers(-1, V, M).astype(np.int32)).cuda()
