@@ -34,7 +34,8 @@ import torch
 
 # tensor ids used in the seed formula config.index * 1000 + id
 _TID = dict(ctx=1, pages=2, q=3, k_blk=4, v_blk=5, k_pages=6, v_pages=7,
-            hidden=8, w=9, mlp=10, drafts=11, sample=12, rl=13)
+            hidden=8, w=9, mlp=10, drafts=11, sample=12, rl=13,
+            draft_q=14, draft_pick=15)
 
 NUM_FEATURES = 8
 
@@ -303,3 +304,28 @@ def rl_batch(seed: int, groups: int, rollouts: int, rounds: int, k: int,
     correct = (rng.random(groups * rollouts) < correct_rate).astype(np.uint8)
     group_off = (np.arange(groups + 1) * rollouts).astype(np.int32)
     return group_off, correct, round_off, match, accept, ell
+
+
+def draft_distributions(cfg: RoundConfig, logits: np.ndarray, noise: float = 1.0,
+                        temperature: float = 1.0) -> np.ndarray:
+    """A stand-in for the draft model's distributions at the K draft
+    positions, for speculative sampling: q_i = softmax((x_{i-1} + noise * eps)
+    / T) with eps ~ N(0, 1), where ``logits`` [B, R, V] are the target's
+    logits of the block rows (whoever computed them) -- a draft that roughly
+    agrees with the target.  Returns float32 [B, K, V]."""
+    x = np.asarray(logits, dtype=np.float64)
+    B, R, V = x.shape
+    rng = np.random.default_rng(seed_of(cfg, "draft_q"))
+    z = (x[:, : R - 1] + noise * rng.standard_normal((B, R - 1, V))) / temperature
+    z -= z.max(axis=-1, keepdims=True)
+    e = np.exp(z)
+    return (e / e.sum(axis=-1, keepdims=True)).astype(np.float32)
+
+
+def sample_from(cfg: RoundConfig, q: np.ndarray, round_index: int = 0) -> np.ndarray:
+    """Draft ids y_hat_i ~ q_i (inverse transform), [B, K] int32."""
+    q = np.asarray(q, dtype=np.float64)
+    rng = np.random.default_rng(seed_of(cfg, "draft_pick") + 7919 * round_index)
+    cdf = np.cumsum(q, axis=-1)
+    r = rng.random(q.shape[:-1] + (1,)) * cdf[..., -1:]
+    return np.minimum(np.sum(cdf < r, axis=-1), q.shape[-1] - 1).astype(np.int32)
