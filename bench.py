@@ -2,16 +2,20 @@
 
 A step is one full round -- L x verify attention, the fused LM head,
 arbitration, accept/commit (with the context restore that lets every step
-verify the same block) -- over one batch of the workload, replayed from CUDA
-graphs.  Metric: verified block-tokens/s = batch * (K+1) / round time.
+verify the same block) -- over one batch of the workload, replayed from a
+CUDA graph.  Metric: verified block-tokens/s = batch * (K+1) / round time.
+The default workload is the largest one: a Llama-3-8B-shaped target, batch
+64, contexts U[8192, 32768], K = 7, 30 % draft mismatches, 32 layers.
 
-  python bench.py [--config qwen3_8b_b1] [--steps K] [--warmup W] [--gpus N]
+  python bench.py [--config NAME] [--steps K] [--warmup W] [--gpus N]
   python bench.py --impl reference      # the CPU oracle on a bounded sample
+  python bench.py --sweep               # the Llama-3-8B batch-64 points:
+                                        # K in {3,5,7} x mismatch 10/30/60 %
 
-One JSON line is printed by rank 0.  Under torchrun every rank runs an
-independent replica of the workload (the round shards by sequence and needs
-no collective); the host-side max over ranks of the timed region gives the
-whole-job throughput.
+One JSON line is printed by rank 0 (one per point with --sweep).  Under
+torchrun every rank runs an independent replica of the workload (the round
+shards by sequence and needs no collective); the host-side max over ranks of
+the timed region gives the whole-job throughput.
 """
 from __future__ import annotations
 
@@ -35,7 +39,8 @@ from paper_2605_24793_gb300 import workload as W  # noqa: E402
 
 METRIC = "verified block-tokens/s (device-timed)"
 UNIT = "block-tokens/s"
-DEFAULT_CONFIG = "qwen3_8b_b1"
+DEFAULT_CONFIG = "llama3_8b_b64_k7_mm30"
+SWEEP = [f"llama3_8b_b64_k{k}_mm{r}" for k in (3, 5, 7) for r in (10, 30, 60)]
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
@@ -139,55 +144,66 @@ def gpu_drafts(cfg, inp) -> np.ndarray:
 
 # ------------------------------------------------------------------ CPU oracle sample
 class OracleSampler:
-    """Times the CPU oracle on a bounded slice of the workload.
+    """Times the CPU oracle on a bounded, seeded sample of one round.
 
-    One sample step runs, for one layer l (cycling), the oracle verify
-    attention of every sequence, the oracle LM head over vocabulary slice l of
-    L (logits and statistics), and the full arbitration, scan and commit of
-    the round.  A full round is L such steps, so the full-round time is
-    estimated as L x the mean step time."""
+    A round is L x B (layer, sequence) attention blocks and their KV commits,
+    the LM head over all M = B * R rows, and the batch's arbitration and
+    scan.  One sample step runs the oracle's verify attention and KV commit
+    of one (layer, sequence) pair from a seeded list, one of L vocabulary
+    slices of the LM head (with its statistics) for all M rows, and the
+    arbitration and acceptance scan of the whole batch.  The full round is
+    extrapolated, not run: the pairs' time per attended key position times
+    the round's key positions (L x sum_b (C_b + R)), plus L x the mean slice
+    time, plus the mean arbitration/scan time."""
 
-    def __init__(self, cfg, inp, draft, max_seqs: int = 64):
+    def __init__(self, cfg, inp, draft, pairs: int = 256, seed: int = 0):
         from oracle import cospec_oracle as O
         self.O = O
         self.cfg = cfg
-        self.draft = draft
-        self.table = inp["page_table_np"]
-        self.ctx = inp["ctx_len_np"]
-        self.hidden = inp["hidden"].cpu()
-        self.w = inp["w"]
         self.inp = inp
+        self.draft = draft
+        self.ctx = inp["ctx_len_np"].astype(np.int64)
+        self.table = inp["page_table_np"]
+        self.hidden = inp["hidden"].cpu()
         self.mlp = inp["mlp"]
-        self.B = cfg.batch
-        self.layer_cache = {}
-        # statistics of the full vocabulary for the arbitration inputs (not timed)
-        self.argmax = None
+        rng = np.random.default_rng(seed)
+        self.pairs = list(zip(rng.integers(0, cfg.layers, pairs).tolist(),
+                              rng.integers(0, cfg.batch, pairs).tolist()))
+        self.n_slices = cfg.layers
+        self.keypos_round = float(cfg.layers * np.sum(self.ctx + cfg.rows))
+        self.rec = []            # per step: (pair seconds, pair key positions, slice s, tail s)
+        self._held = None
 
-    def _layer(self, l):
-        if l not in self.layer_cache:
-            inp, cfg = self.inp, self.cfg
-            lp = 0 if inp["k_pages"].shape[0] == 1 else l
-            pages = np.unique(self.table[self.table >= 0])
-            remap = np.full(inp["num_pages"], -1, dtype=np.int64)
-            remap[pages] = np.arange(len(pages))
-            idx = torch.from_numpy(pages).to(inp["k_pages"].device)
-            self.layer_cache = {l: dict(
-                q=inp["q"][l].cpu(), kb=inp["k_blk"][l].cpu(), vb=inp["v_blk"][l].cpu(),
-                kp=inp["k_pages"][lp].index_select(0, idx).cpu(),
-                vp=inp["v_pages"][lp].index_select(0, idx).cpu(),
-                table=np.where(self.table >= 0, remap[np.clip(self.table, 0, None)], -1))}
-        return self.layer_cache[l]
+    def _pair(self, l, b):
+        """Host copies of layer l's inputs for sequence b (pages relabelled 0..n-1)."""
+        if self._held is not None and self._held[0] == (l, b):
+            return self._held[1]
+        inp = self.inp
+        row = self.table[b]
+        pages = row[row >= 0].astype(np.int64)
+        lp = 0 if inp["k_pages"].shape[0] == 1 else l
+        idx = torch.from_numpy(pages).to(inp["k_pages"].device)
+        d = dict(q=inp["q"][l, b:b + 1].cpu(), kb=inp["k_blk"][l, b:b + 1].cpu(),
+                 vb=inp["v_blk"][l, b:b + 1].cpu(),
+                 kp=inp["k_pages"][lp].index_select(0, idx).cpu(),
+                 vp=inp["v_pages"][lp].index_select(0, idx).cpu(),
+                 table=np.arange(len(pages))[None, :])
+        self._held = ((l, b), d)
+        return d
 
-    def step(self, l):
+    def step(self, i):
         O, cfg = self.O, self.cfg
-        L = cfg.layers
-        d = self._layer(l)
+        l, b = self.pairs[i % len(self.pairs)]
+        sl = i % self.n_slices
+        d = self._pair(l, b)                                  # host copies: not timed
         V = cfg.vocab
-        v0, v1 = (V * l) // L, (V * (l + 1)) // L
-        wslice = self.w[v0:v1].cpu()
+        v0, v1 = (V * sl) // self.n_slices, (V * (sl + 1)) // self.n_slices
+        wslice = self.inp["w"][v0:v1].cpu()
+        P = cfg.page_size
         t0 = time.perf_counter()
-        O.verify_attention(d["q"], d["kb"], d["vb"], d["kp"], d["vp"], d["table"], self.ctx,
-                           cfg.page_size)
+        O.verify_attention(d["q"], d["kb"], d["vb"], d["kp"], d["vp"], d["table"],
+                           self.ctx[b:b + 1], P)
+        t1 = time.perf_counter()
         x = O.lmhead_logits(self.hidden, wslice)
         dfr = np.full((cfg.batch, cfg.rows), -1)
         dfr[:, :cfg.k] = self.draft
@@ -195,24 +211,38 @@ class OracleSampler:
         am, st = O.row_stats(x, dfr.reshape(-1))
         am = am.reshape(cfg.batch, cfg.rows) + v0
         st = st.reshape(cfg.batch, cfg.rows, 5)
+        t2 = time.perf_counter()
         w1, b1, w2, b2 = self.mlp
-        p, a = O.arbitrate(self.draft, am, st, w1, b1, w2, b2, cfg.lam)
+        _, a = O.arbitrate(self.draft, am, st, w1, b1, w2, b2, cfg.lam)
         s, _ = O.accept_scan(self.draft, am, a)
+        t3 = time.perf_counter()
         O.commit_kv(d["kb"].view(torch.int16).numpy()[None], d["vb"].view(torch.int16).numpy()[None],
                     d["kp"].view(torch.int16).numpy()[None], d["vp"].view(torch.int16).numpy()[None],
-                    d["table"], self.ctx, s, cfg.page_size)
-        return time.perf_counter() - t0
+                    d["table"], self.ctx[b:b + 1], s[b:b + 1], P)
+        t4 = time.perf_counter()
+        self.rec.append(((t1 - t0) + (t4 - t3), float(self.ctx[b] + cfg.rows), t2 - t1, t3 - t2))
+        return t4 - t0
 
-    def run(self, budget_s: float, min_steps: int = 1):
-        times = []
+    def round_seconds(self) -> float:
+        r = np.array(self.rec)
+        rate = float(np.mean(r[:, 0] / r[:, 1]))
+        return rate * self.keypos_round + self.n_slices * float(np.mean(r[:, 2])) + float(np.mean(r[:, 3]))
+
+    def describe(self, steps: int) -> str:
+        cfg = self.cfg
+        return (f"{steps} oracle steps, each: verify attention + KV commit of one seeded (layer, "
+                f"sequence) pair, one of {self.n_slices} vocabulary slices of the LM head for all "
+                f"{cfg.m_rows} rows, arbitration + scan of the whole batch; full round extrapolated "
+                f"(not run) = pair time per key position x {self.keypos_round:.0f} key positions "
+                f"+ {self.n_slices} x slice + arbitration/scan = {self.round_seconds():.2f} s")
+
+    def run(self, budget_s: float, min_steps: int = 3):
         t_start = time.perf_counter()
-        l = 0
-        while len(times) < min_steps or time.perf_counter() - t_start < budget_s:
-            times.append(self.step(l % self.cfg.layers))
-            l += 1
-            if len(times) >= self.cfg.layers and time.perf_counter() - t_start >= budget_s:
-                break
-        return times
+        i = 0
+        while i < min_steps or time.perf_counter() - t_start < budget_s:
+            self.step(i)
+            i += 1
+        return i
 
 
 def cpu_threads() -> int:
@@ -228,14 +258,9 @@ def cpu_threads() -> int:
 
 def oracle_baseline(cfg, inp, draft, budget_s: float):
     sampler = OracleSampler(cfg, inp, draft)
-    times = sampler.run(budget_s)
-    round_s = cfg.layers * float(np.mean(times))
-    value = cfg.batch * cfg.rows / round_s
-    sample = (f"{len(times)} oracle steps of 1/{cfg.layers} of a round each (one layer's verify "
-              f"attention for all {cfg.batch} sequences + a 1/{cfg.layers} vocabulary slice of the "
-              f"LM head + arbitration and scan); full round = {cfg.layers} x mean step "
-              f"= {round_s:.2f} s")
-    return value, sample, times
+    n = sampler.run(budget_s)
+    round_s = sampler.round_seconds()
+    return cfg.batch * cfg.rows / round_s, sampler.describe(n)
 
 
 # ------------------------------------------------------------------ reference arm
@@ -243,22 +268,23 @@ def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    cfg = W.CONFIGS[args.config]
-    inp = W.make_round_inputs(cfg, device="cuda" if torch.cuda.is_available() else "cpu")
-    draft = gpu_drafts(cfg, inp) if torch.cuda.is_available() else None
-    if draft is None:
+    cfg = _config(args)
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    inp = W.make_round_inputs(cfg, device=dev)
+    if dev == "cuda":
+        draft = gpu_drafts(cfg, inp)
+    else:
         from oracle import cospec_oracle as O
         x = O.lmhead_logits(inp["hidden"], inp["w"])
         draft = W.synth_drafts(cfg, O.topk_ids(x, 8).reshape(cfg.batch, cfg.rows, 8))
     sampler = OracleSampler(cfg, inp, draft)
     for i in range(args.warmup):
-        sampler.step(i % cfg.layers)
-    times = [sampler.step((args.warmup + i) % cfg.layers) for i in range(args.steps)]
-    round_s = cfg.layers * float(np.mean(times))
+        sampler.step(i)
+    sampler.rec.clear()
+    times = [sampler.step(args.warmup + i) for i in range(args.steps)]
+    round_s = sampler.round_seconds()
     value = cfg.batch * cfg.rows / round_s
-    sample = (f"each step: one layer's oracle verify attention for all {cfg.batch} sequences + a "
-              f"1/{cfg.layers} vocabulary slice of the oracle LM head + arbitration and scan; "
-              f"round time = {cfg.layers} x mean step")
+    sample = sampler.describe(args.steps)
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * float(np.mean(times)), "higher_is_better": True,
@@ -271,49 +297,29 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
-# ------------------------------------------------------------------ our arm
-def main():
-    ap = argparse.ArgumentParser()
-    ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=None)
-    ap.add_argument("--warmup", type=int, default=20)
-    ap.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(W.CONFIGS))
-    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--cpu-budget", type=float, default=12.0)
-    ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--layers", type=int, default=None, help="override the layer count")
-    ap.add_argument("--k", type=int, default=None,
-                    help="override the draft length K (block rows K+1), e.g. 25 as in the paper")
-    ap.add_argument("--temperature", type=float, default=None,
-                    help="stochastic decoding: sample the target candidates at this temperature")
-    args = ap.parse_args()
-    if args.warmup < 3:
-        args.warmup = 3
-    if args.impl == "reference":
-        if args.steps is None:
-            args.steps = 10
-        return run_reference(args)
-
-    from paper_2605_24793_gb300 import replicas
-    world, rank, local_rank = replicas.env_ranks()
-    torch.cuda.set_device(local_rank)
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
-
-    from paper_2605_24793_gb300 import build as BLD
-    from paper_2605_24793_gb300 import cospec as C
-    from paper_2605_24793_gb300.round import VerifyRound
-    C.load_library(BLD.build())
-
+def _config(args):
     cfg = W.CONFIGS[args.config]
     if args.layers:
         cfg = cfg.replace(layers=args.layers)
     if args.k is not None:
         cfg = cfg.replace(k=args.k)
-    inp = W.make_round_inputs(cfg, device="cuda")
+    if args.batch:
+        cfg = cfg.replace(batch=args.batch)
+    return cfg
+
+
+# ------------------------------------------------------------------ our arm
+def measure(cfg, args, env, inp=None, with_cpu=True, with_e2e=True):
+    """Time `cfg`'s round on this GPU; returns the JSON line (rank 0) or None.
+
+    `env` = (world, rank, local_rank, dist).  The round's context is restored
+    at the end, so the inputs can serve another measurement."""
+    from paper_2605_24793_gb300 import cospec as C
+    from paper_2605_24793_gb300 import replicas
+    from paper_2605_24793_gb300.round import VerifyRound
+    world, rank, local_rank, dist = env
+    if inp is None:
+        inp = W.make_round_inputs(cfg, device="cuda")
     draft = gpu_drafts(cfg, inp)
     rnd = VerifyRound(inp, draft, cfg.lam, temperature=args.temperature,
                       seed=W.sample_seed(cfg))
@@ -327,7 +333,8 @@ def main():
     # One graph per round is what a step replays.  Three more graphs of the
     # round's segments -- attention (L launches), LM head, tail (arbitration
     # + commit) -- replayed with events between them give the per-kernel
-    # times of a second timed region.
+    # times of a second timed region.  Graphs of the LM head followed by one
+    # attention launch that may not overlap it give the isolated launch time.
     def cap(fn):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
@@ -346,6 +353,8 @@ def main():
         rnd.commit()
     g_tail = cap(tail)
     g_all = cap(rnd.run)
+    iso_layers = list(range(min(cfg.layers, 4)))
+    g_iso = [cap(lambda l=l: (rnd.lmhead(), rnd.attention(l, kv_stable=False))) for l in iso_layers]
 
     def step():
         g_all.replay()
@@ -358,7 +367,8 @@ def main():
         raise RuntimeError("device error word set during warm-up")
 
     # pick a step count that keeps the timed region near 3 s when none is given
-    if args.steps is None:
+    steps = args.steps
+    if steps is None:
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         with torch.cuda.stream(stream):
             e0.record()
@@ -367,17 +377,21 @@ def main():
             e1.record()
         e1.synchronize()
         per = e0.elapsed_time(e1) / 5
-        args.steps = int(max(20, min(20000, 3000.0 / max(per, 1e-3))))
+        steps = int(max(20, min(20000, 3000.0 / max(per, 1e-3))))
 
-    K = args.steps
+    K = steps
     K2 = min(K, 400)                     # steps of the per-kernel region
+    K3 = max(20, min(200, K2))           # pairs of the isolated-attention region
     e_all = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K2)]
+    ei = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K3)]
     with torch.cuda.stream(stream):
         for _ in range(3):
             g_attn.replay()
             g_lm.replay()
             g_tail.replay()
+        for g in g_iso:
+            g.replay()
     clocks = ClockSampler(local_rank)
     clocks.start()
     time.sleep(0.3)
@@ -402,12 +416,25 @@ def main():
             ev[k][2].record()
             g_tail.replay()
             ev[k][3].record()
+    # third region: LM head alone, then LM head + one attention launch that
+    # starts only after the LM head has ended (no stable-cache overlap); the
+    # difference is the isolated attention launch (cycling over layers)
+    with torch.cuda.stream(stream):
+        for k in range(K3):
+            ei[k][0].record()
+            g_lm.replay()
+            ei[k][1].record()
+            g_iso[k % len(g_iso)].replay()
+            ei[k][2].record()
     torch.cuda.synchronize()
     clk = clocks.stop()
     total_ms = e_all[0].elapsed_time(e_all[1])
     attn_ms = float(np.mean([ev[k][0].elapsed_time(ev[k][1]) for k in range(K2)]))
     lm_ms = float(np.mean([ev[k][1].elapsed_time(ev[k][2]) for k in range(K2)]))
     tail_ms = float(np.mean([ev[k][2].elapsed_time(ev[k][3]) for k in range(K2)]))
+    lm_alone = float(np.mean([ei[k][0].elapsed_time(ei[k][1]) for k in range(K3)]))
+    lm_attn = float(np.mean([ei[k][1].elapsed_time(ei[k][2]) for k in range(K3)]))
+    iso_ms = lm_attn - lm_alone
     total_ms = replicas.max_over_ranks(total_ms, dist, torch.device("cuda", local_rank))
     ms_per_step = total_ms / K
     value = replicas.job_throughput(cfg.batch * cfg.rows, ms_per_step * 1e-3, world)
@@ -425,6 +452,7 @@ def main():
     tflops_peak = float(pk.get("bf16_tflops_sustained", pk["bf16_tflops"]))
     lm_t_hbm = lm_bytes / (hbm * 1e9)
     lm_t_tc = lmhead_flops(cfg) / (tflops_peak * 1e12)
+    seg = attn_ms + lm_ms + tail_ms
     kern = {
         "verify_attn": {"ms_per_launch": attn_launch_ms, "launches_per_step": cfg.layers,
                         "kernel": "tcgen05" if attn_kernel == C.ATTN_TCGEN05 else "mma.sync",
@@ -432,22 +460,32 @@ def main():
                         "bytes_per_launch": a_bytes,
                         "gbs": a_bytes / (attn_launch_ms * 1e-3) / 1e9,
                         "frac_hbm": a_bytes / (attn_launch_ms * 1e-3) / 1e9 / hbm,
-                        "share": attn_ms / (attn_ms + lm_ms + tail_ms)},
+                        "share": attn_ms / seg,
+                        "timing": ("average of the L launches of a round, back to back: each "
+                                   "streams its cache while the previous layer computes")},
+        "verify_attn_isolated": {"ms_per_launch": iso_ms, "bytes_per_launch": a_bytes,
+                                 "gbs": a_bytes / (iso_ms * 1e-3) / 1e9,
+                                 "frac_hbm": a_bytes / (iso_ms * 1e-3) / 1e9 / hbm,
+                                 "layers": len(iso_layers), "pairs": K3,
+                                 "timing": ("one launch after the LM head, with no overlap: "
+                                            "time(LM head + attention) - time(LM head), "
+                                            "each replayed as its own graph")},
         lm_name: {"ms_per_launch": lm_ms, "bytes_per_launch": lm_bytes,
-                                   "flops_per_launch": lmhead_flops(cfg),
-                                   "gbs": lm_bytes / (lm_ms * 1e-3) / 1e9,
-                                   "tflops": lmhead_flops(cfg) / (lm_ms * 1e-3) / 1e12,
-                                   "bound": "hbm" if lm_t_hbm >= lm_t_tc else "tensor",
-                                   "frac_roofline": max(lm_t_hbm, lm_t_tc) / (lm_ms * 1e-3),
-                                   "share": lm_ms / (attn_ms + lm_ms + tail_ms)},
-        "arbitrate+accept_commit": {"ms_per_step": tail_ms,
-                                    "share": tail_ms / (attn_ms + lm_ms + tail_ms)},
+                  "flops_per_launch": lmhead_flops(cfg),
+                  "gbs": lm_bytes / (lm_ms * 1e-3) / 1e9,
+                  "tflops": lmhead_flops(cfg) / (lm_ms * 1e-3) / 1e12,
+                  "bound": "hbm" if lm_t_hbm >= lm_t_tc else "tensor",
+                  "frac_roofline": max(lm_t_hbm, lm_t_tc) / (lm_ms * 1e-3),
+                  "share": lm_ms / seg},
+        "arbitrate+accept_commit": {"ms_per_step": tail_ms, "share": tail_ms / seg},
     }
     if attn_ms >= lm_ms:
         dom = "verify_attn"
         achieved = a_bytes / (attn_launch_ms * 1e-3) / 1e9
         roof = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                "frac": achieved / hbm, "traffic": None}
+                "frac": achieved / hbm, "traffic": None,
+                "isolated": {"achieved": kern["verify_attn_isolated"]["gbs"],
+                             "frac": kern["verify_attn_isolated"]["frac_hbm"]}}
     elif lm_t_hbm >= lm_t_tc:
         dom = lm_name
         achieved = lm_bytes / (lm_ms * 1e-3) / 1e9
@@ -467,43 +505,145 @@ def main():
 
     # ------------------------------------------------------------ end to end (host buffers)
     e2e = None
-    if not args.no_e2e:
+    if with_e2e:
         e2e = end_to_end(cfg, rnd, step, stream, K if K <= 2000 else 2000, dist)
         if dist is None or rank == 0:
             e2e["value"] = world * e2e.pop("per_rank_value")
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        v, sample, _ = oracle_baseline(cfg, inp, draft, args.cpu_budget)
+    if rank == 0 and world == 1 and with_cpu:
+        v, sample = oracle_baseline(cfg, inp, draft, args.cpu_budget)
         cpu = {"value": v, "unit": UNIT, "cores": cpu_threads(), "kind": "oracle", "sample": sample}
+    rnd.restore_context()
+    torch.cuda.synchronize()
 
-    if rank == 0:
-        line = {
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
-            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": cfg.name, "batch": cfg.batch, "k": cfg.k, "rows": cfg.rows,
-                       "layers": cfg.layers, "context": [int(ctx.min()), int(ctx.max())],
-                       "q_heads": cfg.q_heads, "kv_heads": cfg.kv_heads,
-                       "head_dim": cfg.head_dim, "hidden": cfg.hidden, "vocab": cfg.vocab,
-                       "page_size": cfg.page_size, "lambda": cfg.lam,
-                       "decoding": ("greedy" if args.temperature is None
-                                    else f"sampled, T={args.temperature}"),
-                       "parallelism": f"replicas x{world}",
-                       "l2": (f"inputs larger than L2: {(a_bytes * cfg.layers + lm_bytes) / 1e9:.2f}"
-                              " GB streamed per step vs 129 MB L2"),
-                       "graphs": ("one CUDA graph per step; per-kernel times from a second timed "
-                                  f"region of {K2} rounds replaying three graphs (attention, "
-                                  "LM head, arbitration+commit) with events between them")},
-            "roofline": roof, "kernels": kernels_round(kern), "cpu_baseline": cpu, "e2e": e2e,
-            "clocks": clk, "gpu_launches": K * rnd.launches_per_round,
-            "accepted_len_mean": s_mean,
-            "emitted_tokens_per_s": world * cfg.batch * s_mean / (ms_per_step * 1e-3),
-            "accepted_len_of": ("the one synthetic round every step replays (same drafts, "
-                                "context restored); python -m paper_2605_24793_gb300.decode "
-                                "measures it over many rounds"),
-        }
-        print(json.dumps(line), flush=True)
+    if rank != 0:
+        return None
+    return {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": cfg.name, "batch": cfg.batch, "k": cfg.k, "rows": cfg.rows,
+                   "layers": cfg.layers, "context": [int(ctx.min()), int(ctx.max())],
+                   "q_heads": cfg.q_heads, "kv_heads": cfg.kv_heads,
+                   "head_dim": cfg.head_dim, "hidden": cfg.hidden, "vocab": cfg.vocab,
+                   "page_size": cfg.page_size, "lambda": cfg.lam,
+                   "mismatch_rate": cfg.mismatch_rate,
+                   "decoding": ("greedy" if args.temperature is None
+                                else f"sampled, T={args.temperature}"),
+                   "parallelism": f"replicas x{world}",
+                   "l2": (f"inputs larger than L2: {(a_bytes * cfg.layers + lm_bytes) / 1e9:.2f}"
+                          " GB streamed per step vs 129 MB L2"),
+                   "graphs": ("one CUDA graph per step; per-kernel times from a second timed "
+                              f"region of {K2} rounds replaying three graphs (attention, "
+                              "LM head, arbitration+commit) with events between them")},
+        "roofline": roof, "kernels": kernels_round(kern), "cpu_baseline": cpu, "e2e": e2e,
+        "clocks": clk, "gpu_launches": K * rnd.launches_per_round,
+        "accepted_len_mean": s_mean,
+        "emitted_tokens_per_s": world * cfg.batch * s_mean / (ms_per_step * 1e-3),
+        "accepted_len_of": ("the one synthetic round every step replays (same drafts, "
+                            "context restored); python bench.py --sweep and python -m "
+                            "paper_2605_24793_gb300.decode measure it over many rounds"),
+    }
+
+
+def run_sweep(args, env):
+    """Every point of the Llama-3-8B batch-64 workload: K in {3, 5, 7} x draft
+    mismatch rate {10, 30, 60} %.  Per point: the benchmark step (device-timed
+    rounds, per-kernel fractions) and the mean accepted length tau over
+    `--rounds` rounds decoded in a row (Eq. 5)."""
+    from paper_2605_24793_gb300.decode import MultiRoundDecoder
+    names = [n for n in SWEEP if args.points is None or n in args.points]
+    by_k = {}
+    for n in names:
+        by_k.setdefault(W.CONFIGS[n].k, []).append(n)
+    for k, group in by_k.items():
+        base = W.CONFIGS[group[0]]
+        if args.layers:
+            base = base.replace(layers=args.layers)
+        # one set of inputs per K (the mismatch rate changes only the drafts),
+        # with page room for the decoded rounds
+        inp = W.make_round_inputs(base, device="cuda", extra_tokens=args.rounds * base.rows)
+        for n in group:
+            cfg = W.CONFIGS[n].replace(layers=base.layers)
+            inp["cfg"] = cfg
+            line = measure(cfg, args, env, inp=inp, with_cpu=False, with_e2e=False)
+            dec = MultiRoundDecoder(cfg, args.rounds, inputs=inp)
+            res = dec.run()
+            dec.reset()
+            torch.cuda.synchronize()
+            del dec
+            if line is None:
+                continue
+            kk = line["kernels"]
+            lm = kk.get("lmhead_argmax_features") or kk.get("lmhead_sample_features")
+            print(json.dumps({
+                "sweep": "llama3_8b_b64: K x draft mismatch rate",
+                "workload": cfg.name, "k": cfg.k, "mismatch_rate": cfg.mismatch_rate,
+                "batch": cfg.batch, "layers": cfg.layers,
+                "tau": res["tau"], "rounds": res["rounds"],
+                "decode_ms_per_round": res["ms_per_round"],
+                "decode_emitted_tokens_per_s": res["emitted_tokens_per_s"],
+                "block_tokens_per_s": line["value"], "ms_per_step": line["ms_per_step"],
+                "steps": line["steps"],
+                "attention_us_per_launch": 1e3 * kk["verify_attn"]["ms_per_launch"],
+                "attention_frac_hbm": kk["verify_attn"]["frac_hbm"],
+                "attention_isolated_frac_hbm": kk["verify_attn_isolated"]["frac_hbm"],
+                "lmhead_us": 1e3 * lm["ms_per_launch"], "lmhead_bound": lm["bound"],
+                "lmhead_frac_roofline": lm["frac_roofline"],
+                "device_error": res["device_error"], "clocks": line["clocks"]}), flush=True)
+        del inp
+        torch.cuda.empty_cache()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=None)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(W.CONFIGS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--layers", type=int, default=None, help="override the layer count")
+    ap.add_argument("--batch", type=int, default=None,
+                    help="override the batch (a smaller case of the same shapes)")
+    ap.add_argument("--k", type=int, default=None,
+                    help="override the draft length K (block rows K+1), e.g. 25 as in the paper")
+    ap.add_argument("--temperature", type=float, default=None,
+                    help="stochastic decoding: sample the target candidates at this temperature")
+    ap.add_argument("--sweep", action="store_true",
+                    help="the Llama-3-8B batch-64 points (K x mismatch rate), one line each")
+    ap.add_argument("--points", nargs="+", default=None, help="subset of the sweep's workloads")
+    ap.add_argument("--rounds", type=int, default=32, help="decoded rounds per sweep point")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        if args.steps is None:
+            args.steps = 10
+        return run_reference(args)
+
+    from paper_2605_24793_gb300 import replicas
+    world, rank, local_rank = replicas.env_ranks()
+    torch.cuda.set_device(local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+
+    from paper_2605_24793_gb300 import build as BLD
+    from paper_2605_24793_gb300 import cospec as C
+    C.load_library(BLD.build())
+    env = (world, rank, local_rank, dist)
+    if args.sweep:
+        run_sweep(args, env)
+    else:
+        line = measure(_config(args), args, env, with_cpu=not args.no_cpu_baseline,
+                       with_e2e=not args.no_e2e)
+        if line is not None:
+            print(json.dumps(line), flush=True)
     if dist:
         dist.barrier()
         dist.destroy_process_group()
@@ -511,10 +651,7 @@ def main():
 
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture
 # (profiles/), keyed by (workload, kernel); an entry is removed when its
-# kernel changes after the capture.  The attention entries (qwen3_8b_b1
-# 16918528, qwen3_8b_b16 304239360, qwen3_32b_b32 1362598144 bytes) were
-# removed when both attention kernels changed how they issue the cluster
-# merge's copies; they come back with the next capture.
+# kernel changes after the capture.
 TRAFFIC = {
     ("qwen3_8b_b1", "lmhead_argmax_features"): 1248011008.0,
 }

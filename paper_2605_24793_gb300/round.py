@@ -99,14 +99,16 @@ class VerifyRound:
         """Reset ctx_len to the round's starting context (device copy)."""
         self.ctx_len.copy_(self.ctx0, non_blocking=True)
 
-    def attention(self, l: int) -> torch.Tensor:
+    def attention(self, l: int, kv_stable: Optional[bool] = None) -> torch.Tensor:
+        """Layer l's verify attention.  ``kv_stable`` (default: l > 0) lets the
+        launch stream its cache before the previous kernel ends."""
         pl = 0 if self.k_pages.shape[0] == 1 else l
         out = self.attn_out[l if self.attn_out.shape[0] > 1 else 0]
         # Layers after the first follow another attention launch, which writes
         # neither the context lengths, the page table nor the cached pages.
         return C.verify_attn(self.q[l], self.k_blk[l], self.v_blk[l], self.k_pages[pl],
                              self.v_pages[pl], self.page_table, self.ctx_len, out, self.max_ctx,
-                             kv_stable=l > 0)
+                             kv_stable=(l > 0) if kv_stable is None else kv_stable)
 
     def lmhead(self):
         if self.temperature is not None:

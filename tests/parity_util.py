@@ -32,22 +32,43 @@ def assert_close(got, ref, what: str, abs_tol: float = TOL_ABS, rel_tol: float =
     return float(err.max()) if err.size else 0.0
 
 
-def tie_affected(ref_stats, ref_draft, ref_argmax, ref_p, s_ref, s_gpu, lam, margin=None):
-    """Per-sequence tie flags.  ref_stats [B,R,5], ref_draft [B,K],
-    ref_argmax [B,R], ref_p [B,K], s_* [B].  ``margin`` [B,R] overrides the
-    top-1/top-2 logit gap (for sampled candidates: the gap of the perturbed
-    keys)."""
+def tie_positions(ref_stats, ref_draft, ref_argmax, ref_p, s_ref, s_gpu, lam, margin=None):
+    """Near-tie positions of each sequence among those that decide its round:
+    rows 0..min(K, max(s_oracle, s_gpu)) whose oracle top-1/top-2 margin is
+    below TIE, and evaluated mismatches whose policy probability is within
+    TIE of lambda.  ref_stats [B,R,5], ref_draft [B,K], ref_argmax [B,R],
+    ref_p [B,K], s_* [B].  ``margin`` [B,R] overrides the top-1/top-2 logit
+    gap (for sampled candidates: the gap of the perturbed keys).  Returns an
+    int array [B] of counts."""
     B, R = ref_argmax.shape
     K = R - 1
     if margin is None:
         margin = ref_stats[:, :, 0] - ref_stats[:, :, 1]
-    flags = np.zeros(B, dtype=bool)
+    counts = np.zeros(B, dtype=np.int64)
     for b in range(B):
         reach = min(K, int(max(s_ref[b], s_gpu[b])))
-        if np.any(margin[b, : reach + 1] < TIE):
-            flags[b] = True
-            continue
+        counts[b] += int(np.sum(margin[b, : reach + 1] < TIE))
         for i in range(1, reach + 1):
             if i <= K and ref_draft[b, i - 1] != ref_argmax[b, i - 1] and abs(ref_p[b, i - 1] - lam) < TIE:
-                flags[b] = True
-    return flags
+                counts[b] += 1
+    return counts
+
+
+def tie_affected(ref_stats, ref_draft, ref_argmax, ref_p, s_ref, s_gpu, lam, margin=None):
+    """Per-sequence tie flags: a sequence with any near-tie position
+    (tie_positions) has its discrete outputs excluded from the bit-exact
+    comparison."""
+    return tie_positions(ref_stats, ref_draft, ref_argmax, ref_p, s_ref, s_gpu, lam, margin) > 0
+
+
+# (test, workload, tie-affected sequences, sequences, near-tie positions) of
+# every parity test that counts ties; printed at the end of the session and,
+# when COSPEC_PARITY_REPORT names a file, written there as JSON.
+TIE_REPORT = []
+
+
+def report_ties(test: str, workload: str, counts) -> None:
+    counts = np.asarray(counts)
+    TIE_REPORT.append({"test": test, "workload": workload,
+                       "tie_affected_sequences": int(np.sum(counts > 0)),
+                       "sequences": int(counts.size), "tie_positions": int(np.sum(counts))})

@@ -11,7 +11,7 @@ from paper_2605_24793_gb300 import cospec as C
 from paper_2605_24793_gb300 import workload as W
 from paper_2605_24793_gb300.decode import MultiRoundDecoder
 
-from .parity_util import tie_affected
+from .parity_util import report_ties, tie_positions
 
 pytestmark = pytest.mark.gpu
 
@@ -42,7 +42,9 @@ def test_rounds_match_oracle_round_by_round(k, rounds, lam):
     tie_seqs = np.zeros(cfg.batch, dtype=bool)
     for r in range(rounds):
         ref = O.cospec_round(state, drafts[r], lam, with_attention=False)
-        tie_seqs |= tie_affected(ref["stats"], drafts[r], ref["argmax"], ref["p"], ref["s"], s_gpu[r], lam)
+        ties = tie_positions(ref["stats"], drafts[r], ref["argmax"], ref["p"], ref["s"], s_gpu[r], lam)
+        report_ties("multi-round parity", f"{cfg.name} K={k} lambda={lam} round {r}", ties)
+        tie_seqs |= ties > 0
         ok = ~tie_seqs
         assert np.array_equal(s_gpu[r][ok], ref["s"][ok]), f"round {r}"
         assert np.array_equal(em_gpu[r][ok], ref["emitted"][ok]), f"round {r}"
@@ -86,8 +88,10 @@ def test_sampled_rounds_match_oracle_round_by_round():
     for r in range(rounds):
         ref = O.cospec_round(state, drafts[r], lam, with_attention=False,
                              sample_seed=W.sample_seed(cfg, r), temperature=T)
-        tie_seqs |= tie_affected(ref["stats"], drafts[r], ref["argmax"], ref["p"], ref["s"],
-                                 s_gpu[r], lam, margin=ref["key_margin"])
+        ties = tie_positions(ref["stats"], drafts[r], ref["argmax"], ref["p"], ref["s"],
+                             s_gpu[r], lam, margin=ref["key_margin"])
+        report_ties("sampled multi-round parity", f"{cfg.name} K={k} T={T} round {r}", ties)
+        tie_seqs |= ties > 0
         ok = ~tie_seqs
         assert np.array_equal(s_gpu[r][ok], ref["s"][ok]), f"round {r}"
         assert np.array_equal(em_gpu[r][ok], ref["emitted"][ok]), f"round {r}"

@@ -1,7 +1,6 @@
 """Parity of the CUDA path (through the C ABI) with the CPU oracle on seeded
 inputs small enough for the oracle, spanning several tiles, ragged tails and
 the degenerate cases (empty context, K = 0, single / many KV splits)."""
-import ctypes
 import math
 
 import numpy as np
@@ -14,7 +13,7 @@ from paper_2605_24793_gb300 import cospec as C
 from paper_2605_24793_gb300 import workload as W
 from paper_2605_24793_gb300.round import VerifyRound
 
-from .parity_util import assert_close, tie_affected
+from .parity_util import assert_close, report_ties, tie_positions
 
 pytestmark = pytest.mark.gpu
 
@@ -425,7 +424,9 @@ def _check_round(cfg, draft, ref, rnd, lam):
     st = rnd.stats.cpu().numpy().reshape(B, R, 5)
     assert_close(st, ref["stats"], "lm-head stats")
     s_gpu = rnd.accept_len.cpu().numpy()
-    tie = tie_affected(ref["stats"], draft, ref["argmax"], ref["p"], ref["s"], s_gpu, lam)
+    ties = tie_positions(ref["stats"], draft, ref["argmax"], ref["p"], ref["s"], s_gpu, lam)
+    report_ties("round parity", f"{cfg.name} K={K} lambda={lam}", ties)
+    tie = ties > 0
     ok = ~tie
     am = rnd.argmax.cpu().numpy().reshape(B, R)
     assert np.array_equal(am[ok], ref["argmax"][ok])
@@ -640,8 +641,10 @@ def test_tiny_sampled_round_matches_oracle(T):
     ref = O.cospec_round(hostd, draft, cfg.lam, with_attention=False, with_commit=False,
                          sample_seed=seed, temperature=T)
     s_gpu = rnd.accept_len.cpu().numpy()
-    tie = tie_affected(ref["stats"], draft, ref["argmax"], ref["p"], ref["s"], s_gpu, cfg.lam,
-                       margin=ref["key_margin"])
+    ties = tie_positions(ref["stats"], draft, ref["argmax"], ref["p"], ref["s"], s_gpu, cfg.lam,
+                         margin=ref["key_margin"])
+    report_ties("sampled round parity", f"{cfg.name} T={T}", ties)
+    tie = ties > 0
     ok = ~tie
     assert np.array_equal(s_gpu[ok], ref["s"][ok])
     assert np.array_equal(rnd.emitted.cpu().numpy().reshape(cfg.batch, -1)[ok], ref["emitted"][ok])
