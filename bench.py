@@ -651,9 +651,13 @@ def main():
 
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture
 # (profiles/), keyed by (workload, kernel); an entry is removed when its
-# kernel changes after the capture.
+# kernel changes after the capture.  Llama batch 64: the mean of two
+# full-size launches; Qwen3-32B: one launch of a two-layer run (the
+# per-layer shapes of the full workload).
 TRAFFIC = {
-    ("qwen3_8b_b1", "lmhead_argmax_features"): 1248011008.0,
+    ("llama3_8b_b64_k7_mm30", "verify_attn"): 5224817280.0,
+    ("qwen3_8b_b1", "verify_attn"): 16918528.0,
+    ("qwen3_32b_b32", "verify_attn"): 1362594304.0,
 }
 
 
