@@ -237,6 +237,25 @@ COSPEC_API int cospec_lmhead_sample_features(int M, int d, int V, const uint16_t
                                              int32_t* sample, float* stats, void* ws,
                                              size_t ws_bytes, void* stream);
 
+/* The LM head for speculative sampling at temperature T (the exact-match
+ * baseline of Sec. 3.1 "Stochastic decoding" / App. C.3, see
+ * cospec_sps_accept): the scaled logits x / T are written out, and the
+ * statistics are those of x / T.
+ *
+ *    logits   float32 [M, V]: logits[m][v] = (hidden[m] . W[v]) / T (4-byte aligned)
+ *    argmax   int32 [M]: lowest id among the maximal logits (as the greedy call)
+ *    stats    float32 [M, 5]: as the greedy call, for the scaled logits x / T
+ *             (stats[m][2] = log sum_v exp(x_v / T); stats[m][4] = x[draft] / T)
+ *    temperature > 0 and finite; other arguments and the workspace as for
+ *    cospec_lmhead_argmax_features.
+ * The M x V logits are written to memory (M * V * 4 bytes); the greedy and
+ * sampling calls never write them. */
+COSPEC_API int cospec_lmhead_logits_features(int M, int d, int V, const uint16_t* hidden,
+                                             const uint16_t* w, const int32_t* draft_for_row,
+                                             float temperature, int32_t* argmax, float* stats,
+                                             float* logits, void* ws, size_t ws_bytes,
+                                             void* stream);
+
 /* Same computation and outputs as cospec_lmhead_argmax_features, for callers
  * that cannot allocate device memory or hand this library a workspace -- for
  * example a serving engine that reserves nearly all HBM for its KV cache and
@@ -258,6 +277,47 @@ COSPEC_API int cospec_lmhead_argmax_features_noalloc(int M, int d, int V, const 
                                                      const uint16_t* w,
                                                      const int32_t* draft_for_row,
                                                      int32_t* argmax, float* stats, void* stream);
+
+/* ------------------------------------------------------------------------ */
+/* 2b. Speculative-sampling acceptance: the distribution-preserving baseline
+ *    that the paper compares against at T = 1 (Sec. 3.1 "Stochastic
+ *    decoding"; App. C.3: standard speculative sampling with acceptance-ratio
+ *    correction, Leviathan et al. 2023 / Chen et al. 2023).  It replaces the
+ *    arbitration step of a CoSpec round.
+ *
+ *    With p_i = softmax(x_{i-1} / T) (block row i-1's scaled logits) and the
+ *    draft's distribution q_i at draft position i:
+ *      ratio[b][i-1] = min(1, p_i(y_hat_i) / q_i(y_hat_i))   (1 when q_i(y_hat_i) = 0)
+ *      y_hat_i is accepted iff u * q_i(y_hat_i) < p_i(y_hat_i), u the uniform of
+ *        (b, i): output word 0 of Philox4x32-10 at counter (i - 1, b, 1, 0)
+ *        under the key (seed mod 2^32, floor(seed / 2^32)),
+ *        u = (floor(r / 2^9) + 0.5) / 2^23;
+ *      at the first rejection i*, target[b][i*-1] = a draw from
+ *        max(0, p_{i*} - q_{i*}) (renormalised); with no rejection,
+ *        target[b][K] = a draw from p_{K+1}.  Both draws are Gumbel-max,
+ *        argmax_v (log w(v) + g_{m,v}), with the Gumbel noise of block row
+ *        m = b (K + 1) + row that cospec_lmhead_sample_features uses (a
+ *        residual with no positive entry, possible only through rounding,
+ *        falls back to p).
+ *    accept[b][i-1] = 1 before the stop row, 0 from it on; target[b][j] =
+ *    y_hat_{j+1} before the stop row, -1 after it.  Passing (target, accept)
+ *    as (argmax, accept) to cospec_accept_commit then yields the accepted
+ *    length, the emitted tokens and the KV commit.
+ *
+ *    draft  int32 [B, K]
+ *    stats  float32 [B*(K+1), 5] and logits float32 [B*(K+1), V] from
+ *           cospec_lmhead_logits_features at temperature T
+ *    q      float32 [B, K, V]: the draft's distribution at every position
+ *    seed   DEVICE pointer to one uint64 (8-byte aligned), read when the kernel runs
+ *    target int32 [B, K+1]; accept uint8 [B, K]; ratio float32 [B, K]
+ *    ws     >= cospec_sps_workspace(B) bytes, 16-byte aligned (no initialisation)
+ *    Supported: 0 <= K <= 31 (draft, q, accept, ratio may be NULL when K = 0).
+ *    A draft id outside [0, V) sets COSPEC_DEVERR_TOKEN and is rejected. */
+COSPEC_API size_t cospec_sps_workspace(int B);
+COSPEC_API int cospec_sps_accept(int B, int K, int V, const int32_t* draft, const float* stats,
+                                 const float* logits, const float* q, const uint64_t* seed,
+                                 int32_t* target, uint8_t* accept, float* ratio, void* ws,
+                                 size_t ws_bytes, void* stream);
 
 /* ------------------------------------------------------------------------ */
 /* 3. Arbitration at draft/target mismatches (Sec. 3.3).

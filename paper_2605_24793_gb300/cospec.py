@@ -24,7 +24,8 @@ EXPORTED = ("cospec_status_string", "cospec_last_cuda_error", "cospec_get_device
             "cospec_verify_attn", "cospec_lmhead_workspace", "cospec_lmhead_argmax_features",
             "cospec_arbitrate", "cospec_accept_commit", "cospec_lmhead_argmax_features_noalloc",
             "cospec_lmhead_sample_features", "cospec_verify_attn_plan", "cospec_rl_workspace",
-            "cospec_rl_advantages", "cospec_verify_attn_plan_model")
+            "cospec_rl_advantages", "cospec_verify_attn_plan_model",
+            "cospec_lmhead_logits_features", "cospec_sps_workspace", "cospec_sps_accept")
 
 
 class AttnDims(ctypes.Structure):
@@ -87,6 +88,11 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "cospec_lmhead_argmax_features_noalloc": (_i, [_i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp]),
         "cospec_lmhead_sample_features": (_i, [_i, _i, _i, _vp, _vp, _vp, _f, _vp, _vp, _vp, _vp,
                                                _sz, _vp]),
+        "cospec_lmhead_logits_features": (_i, [_i, _i, _i, _vp, _vp, _vp, _f, _vp, _vp, _vp, _vp,
+                                               _sz, _vp]),
+        "cospec_sps_workspace": (_sz, [_i]),
+        "cospec_sps_accept": (_i, [_i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
+                                   _vp]),
         "cospec_arbitrate": (_i, [_i, _i, _vp, _vp, _vp, _i, _vp, _vp, _vp, _f, _f, _i, _vp, _vp, _vp]),
         "cospec_accept_commit": (_i, [_i, _i, _i, _PDIMS, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                       ctypes.c_longlong, _vp, _vp, _vp, _vp, _vp]),
@@ -308,6 +314,63 @@ def lmhead_sample_features(hidden, w, draft_for_row, temperature: float, seed, s
         M, d, V, _ptr(hidden), _ptr(w), _ptr(draft_for_row), float(temperature), _ptr(seed),
         _ptr(sample), _ptr(stats), _ptr(ws), ws.numel(), _stream(stream)))
     return sample, stats
+
+
+def lmhead_logits_features(hidden, w, draft_for_row, temperature: float, argmax, stats, logits,
+                           ws, stream=None):
+    """LM head for speculative sampling at temperature T: logits [M, V] fp32
+    receives x / T, stats [M, 5] the statistics of x / T, argmax [M] the
+    argmax."""
+    _req(hidden, torch.bfloat16, "hidden", 2)
+    _req(w, torch.bfloat16, "w", 2)
+    _req(draft_for_row, torch.int32, "draft_for_row", 1)
+    _req(argmax, torch.int32, "argmax", 1)
+    _req(stats, torch.float32, "stats", 2)
+    _req(logits, torch.float32, "logits", 2)
+    _req(ws, torch.uint8, "ws", 1)
+    M, d = hidden.shape
+    V = w.shape[0]
+    if (w.shape[1] != d or draft_for_row.numel() != M or argmax.numel() != M
+            or tuple(stats.shape) != (M, 5) or tuple(logits.shape) != (M, V)):
+        raise ValueError("inconsistent LM-head shapes")
+    _same_device(hidden, w, draft_for_row, argmax, stats, logits, ws)
+    _check(load_library().cospec_lmhead_logits_features(
+        M, d, V, _ptr(hidden), _ptr(w), _ptr(draft_for_row), float(temperature), _ptr(argmax),
+        _ptr(stats), _ptr(logits), _ptr(ws), ws.numel(), _stream(stream)))
+    return argmax, stats, logits
+
+
+def new_sps_workspace(B: int, device="cuda") -> torch.Tensor:
+    return torch.empty(max(1, int(load_library().cospec_sps_workspace(B))), dtype=torch.uint8,
+                       device=device)
+
+
+def sps_accept(draft, stats, logits, q, seed, target, accept, ratio, ws, stream=None):
+    """Speculative-sampling acceptance (the exact-match baseline at a
+    temperature): draft [B, K], stats [B*(K+1), 5] and logits [B*(K+1), V]
+    of x / T, q [B, K, V] the draft's distributions, seed an int64 device
+    scalar; fills target [B, K+1], accept [B, K], ratio [B, K]."""
+    _req(draft, torch.int32, "draft", 2)
+    _req(stats, torch.float32, "stats", 2)
+    _req(logits, torch.float32, "logits", 2)
+    _req(q, torch.float32, "q", 3)
+    _req(seed, torch.int64, "seed")
+    _req(target, torch.int32, "target")
+    _req(accept, torch.uint8, "accept")
+    _req(ratio, torch.float32, "ratio")
+    _req(ws, torch.uint8, "ws", 1)
+    B, K = draft.shape
+    R = K + 1
+    V = logits.shape[1]
+    if (seed.numel() != 1 or tuple(stats.shape) != (B * R, 5) or logits.shape[0] != B * R
+            or tuple(q.shape) != (B, K, V) or target.numel() != B * R or accept.numel() != B * K
+            or ratio.numel() != B * K):
+        raise ValueError("inconsistent speculative-sampling shapes")
+    _same_device(draft, stats, logits, q, seed, target, accept, ratio, ws)
+    _check(load_library().cospec_sps_accept(
+        B, K, V, _ptr(draft), _ptr(stats), _ptr(logits), _ptr(q), _ptr(seed), _ptr(target),
+        _ptr(accept), _ptr(ratio), _ptr(ws), ws.numel(), _stream(stream)))
+    return target, accept, ratio
 
 
 def lmhead_argmax_features_noalloc(hidden, w, draft_for_row, argmax, stats, stream=None):

@@ -351,6 +351,67 @@ COSPEC_API int cospec_lmhead_sample_features(int M, int d, int V, const uint16_t
                                  1.0f / temperature));
 }
 
+COSPEC_API int cospec_lmhead_logits_features(int M, int d, int V, const uint16_t* hidden,
+                                             const uint16_t* w, const int32_t* draft_for_row,
+                                             float temperature, int32_t* argmax, float* stats,
+                                             float* logits, void* ws, size_t ws_bytes,
+                                             void* stream) {
+  CS_CHECK_ARG(M >= 0 && d > 0 && V > 0);
+  CS_CHECK_ARG(temperature > 0.f && isfinite(temperature) && isfinite(1.0f / temperature));
+  if (M == 0) return COSPEC_OK;
+  CS_CHECK_ARG(hidden && w && draft_for_row && argmax && stats && logits);
+  if (d % 64 != 0) return COSPEC_ERR_UNSUPPORTED;
+  if ((long long)V > 0x7fffff00LL) return COSPEC_ERR_UNSUPPORTED;
+  CS_CHECK_ARG(aligned16(hidden) && aligned16(w) && (reinterpret_cast<uintptr_t>(logits) & 3u) == 0);
+  const int sms = device_num_sms();
+  if (sms <= 0) return cuda_lookup_failed();
+  const LmheadPlan pl = plan_lmhead(M, d, V, sms);
+  if (!ws || ws_bytes < pl.ws_bytes || !aligned16(ws)) return COSPEC_ERR_WORKSPACE;
+  int* err = device_error_word();
+  if (!err) return cuda_lookup_failed();
+  return cuda_status(launch_lmhead(M, d, V, reinterpret_cast<const __nv_bfloat16*>(hidden),
+                                   reinterpret_cast<const __nv_bfloat16*>(w), draft_for_row,
+                                   argmax, stats, ws, pl, err, static_cast<cudaStream_t>(stream),
+                                   nullptr, 1.0f / temperature, logits));
+}
+
+// ---------------------------------------------------------------- speculative sampling
+COSPEC_API size_t cospec_sps_workspace(int B) {
+  if (B < 1) return 0;
+  return (size_t)B * SPS_MAX_SLICES * 16 + (size_t)B * 4 + 256;
+}
+
+COSPEC_API int cospec_sps_accept(int B, int K, int V, const int32_t* draft, const float* stats,
+                                 const float* logits, const float* q, const uint64_t* seed,
+                                 int32_t* target, uint8_t* accept, float* ratio, void* ws,
+                                 size_t ws_bytes, void* stream) {
+  CS_CHECK_ARG(B >= 0 && K >= 0 && V > 0);
+  if (K > 31) return COSPEC_ERR_UNSUPPORTED;
+  if (B == 0) return COSPEC_OK;
+  CS_CHECK_ARG(stats && logits && seed && target);
+  CS_CHECK_ARG(K == 0 || (draft && q && accept && ratio));
+  CS_CHECK_ARG((reinterpret_cast<uintptr_t>(seed) & 7u) == 0);
+  if (!ws || ws_bytes < cospec_sps_workspace(B) || !aligned16(ws)) return COSPEC_ERR_WORKSPACE;
+  const int sms = device_num_sms();
+  if (sms <= 0) return cuda_lookup_failed();
+  int* err = device_error_word();
+  if (!err) return cuda_lookup_failed();
+  SpsArgs a{};
+  a.B = B;
+  a.K = K;
+  a.V = V;
+  a.draft = draft;
+  a.stats = stats;
+  a.logits = logits;
+  a.q = q;
+  a.seed = reinterpret_cast<const unsigned long long*>(seed);
+  a.target = target;
+  a.accept = accept;
+  a.ratio = ratio;
+  a.ws = ws;
+  return cuda_status(launch_sps(a, sms, err, static_cast<cudaStream_t>(stream)));
+}
+
 // ---------------------------------------------------------------- arbitration
 COSPEC_API int cospec_arbitrate(int B, int K, const int32_t* draft, const int32_t* argmax,
                                 const float* stats, int mlp_hidden, const float* w1,

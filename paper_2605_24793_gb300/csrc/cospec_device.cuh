@@ -312,4 +312,36 @@ CS_DEV int sequence_by_rank(const int32_t* ctx_len, int B, int z, volatile int* 
 }
 
 
+// Philox4x32-10: ten rounds of two 32x32 -> 64-bit products by the
+// multipliers 0xD2511F53 / 0xCD9E8D57, the key advanced by the Weyl
+// increments 0x9E3779B9 / 0xBB67AE85 between rounds.
+CS_DEV uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r) {
+      k0 += 0x9E3779B9u;
+      k1 += 0xBB67AE85u;
+    }
+    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+  }
+  return c;
+}
+
+// Standard Gumbel variate g = -log(E), E = -log(u) ~ Exp(1), from 32 random
+// bits: u = (floor(r / 2^9) + 0.5) / 2^23 is an odd multiple of 2^-24 in (0, 1),
+// exact in float32, and so is w = 1 - u.  Near u = 1 (w < 1/64) E comes from
+// the series -log(1 - w) = w + w^2/2 + w^3/3 + w^4/4 + ..., whose truncation
+// is below 1e-8 relative there; elsewhere |log u| > 1/64 and the fast
+// logarithm's absolute error (about 4e-7) is at most ~3e-5 relative.  The
+// largest keys, which decide the sample, come from the series branch.
+CS_DEV float gumbel_of(uint32_t r) {
+  const float u = ((float)(r >> 9) + 0.5f) * 1.1920928955078125e-7f;
+  const float w = 1.f - u;
+  const float e_series = w * fmaf(w, fmaf(w, fmaf(w, 0.25f, 0.333333343f), 0.5f), 1.f);
+  const float e = (w < 0.015625f) ? e_series : -__logf(u);
+  return -__logf(e);
+}
+
 }  // namespace cospec

@@ -115,7 +115,24 @@ cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
                           const __nv_bfloat16* w, const int32_t* draft_for_row, int32_t* argmax,
                           float* stats, void* ws, const LmheadPlan& plan, int* err,
                           cudaStream_t stream, const unsigned long long* seed = nullptr,
-                          float inv_temp = 1.f);
+                          float inv_temp = 1.f, float* logits = nullptr);
+
+// ---------------------------------------------------------------- speculative sampling
+constexpr int SPS_MAX_SLICES = 64;   // vocabulary slices (CTAs) per sequence
+struct SpsArgs {
+  int B, K, V;
+  const int32_t* draft;
+  const float* stats;
+  const float* logits;
+  const float* q;
+  const unsigned long long* seed;
+  int32_t* target;
+  uint8_t* accept;
+  float* ratio;
+  void* ws;
+};
+int sps_slices(int B, int V, int num_sms);
+cudaError_t launch_sps(const SpsArgs& a, int num_sms, int* err, cudaStream_t stream);
 
 // ---------------------------------------------------------------- arbitration
 cudaError_t launch_arbitrate(int B, int K, const int32_t* draft, const int32_t* argmax,

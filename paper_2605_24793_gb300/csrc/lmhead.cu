@@ -30,6 +30,11 @@
 // counter (v, m / 4, 0, 0), output m % 4, so a thread that owns vocab id v and
 // four consecutive rows makes one generator call.  The tuple then carries the
 // best key k and i becomes its id; m, sec, s, t stay statistics of the logits.
+//
+// Speculative sampling (the distribution-preserving baseline at temperature
+// T, Sec. 3.1) needs the target's whole distribution at the row where a draft
+// token is rejected, so a third mode (MODE_LOGITS) scales the logits by 1 / T,
+// writes them out ([M, V] fp32) and keeps the statistics of the scaled logits.
 #include <cuda.h>
 #include <math.h>
 
@@ -110,38 +115,6 @@ CS_DEV Stat stat_of(float x, float k, int v) {
   return Stat{x, v, -INFINITY, (x == -INFINITY) ? 0.f : 1.f, 0.f, k};
 }
 
-// Philox4x32-10: ten rounds of two 32x32 -> 64-bit products by the
-// multipliers 0xD2511F53 / 0xCD9E8D57, the key advanced by the Weyl
-// increments 0x9E3779B9 / 0xBB67AE85 between rounds.
-CS_DEV uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
-#pragma unroll
-  for (int r = 0; r < 10; ++r) {
-    if (r) {
-      k0 += 0x9E3779B9u;
-      k1 += 0xBB67AE85u;
-    }
-    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
-    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
-    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
-  }
-  return c;
-}
-
-// Standard Gumbel variate g = -log(E), E = -log(u) ~ Exp(1), from 32 random
-// bits: u = (floor(r / 2^9) + 0.5) / 2^23 is an odd multiple of 2^-24 in (0, 1),
-// exact in float32, and so is w = 1 - u.  Near u = 1 (w < 1/64) E comes from
-// the series -log(1 - w) = w + w^2/2 + w^3/3 + w^4/4 + ..., whose truncation
-// is below 1e-8 relative there; elsewhere |log u| > 1/64 and the fast
-// logarithm's absolute error (about 4e-7) is at most ~3e-5 relative.  The
-// largest keys, which decide the sample, come from the series branch.
-CS_DEV float gumbel_of(uint32_t r) {
-  const float u = ((float)(r >> 9) + 0.5f) * 1.1920928955078125e-7f;
-  const float w = 1.f - u;
-  const float e_series = w * fmaf(w, fmaf(w, fmaf(w, 0.25f, 0.333333343f), 0.5f), 1.f);
-  const float e = (w < 0.015625f) ? e_series : -__logf(u);
-  return -__logf(e);
-}
-
 // Reduce 16 columns held by every lane of a warp (lane l holds vocab id
 // base + l) so that lanes 2c and 2c+1 end with column c reduced over all 32
 // lanes.  Each butterfly level exchanges half of the remaining columns, so a
@@ -203,7 +176,8 @@ struct LmParams {
   int* part_idx;                 // [gridDim.x][n_rows]
   float* part_k;                 // [gridDim.x][n_rows], KEYED only
   const unsigned long long* seed;  // KEYED only: Philox key (low word, high word)
-  float inv_temp;                // KEYED only: 1 / T
+  float inv_temp;                // KEYED and LOGITS: 1 / T
+  float* logits;                 // LOGITS only: [M][V] x / T
   int row0, n_rows, n_mma;
   int d, V, num_tiles, stages;
   uint32_t tmem_cols;
@@ -231,10 +205,14 @@ __host__ __device__ inline SmemLayout lm_layout(int stages, int n_mma, bool keye
   return L;
 }
 
-template <bool KEYED>
+enum : int { MODE_GREEDY = 0, MODE_KEYED = 1, MODE_LOGITS = 2 };
+
+template <int MODE>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     lmhead_kernel(const __grid_constant__ CUtensorMap tmap_w,
                   const __grid_constant__ CUtensorMap tmap_h, const LmParams p) {
+  constexpr bool KEYED = MODE == MODE_KEYED;
+  constexpr bool LOGITS = MODE == MODE_LOGITS;
   extern __shared__ uint8_t smem_raw[];
   // TMA with 128B swizzle and the UMMA descriptors need 1024-byte alignment.
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -465,6 +443,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       for (int ch = half; ch < nchunks; ch += EPI_WARPS / 4) {
         float x[16];
         tmem_ld16(tbase + (uint32_t)(ch * 16), x);
+        if (LOGITS) {
+          // x / T, written row by row: the warp's 32 lanes hold 32 consecutive
+          // vocabulary ids of one row, so each store is one 128-byte line
+#pragma unroll
+          for (int c = 0; c < 16; ++c) {
+            x[c] *= p.inv_temp;
+            const int col = ch * 16 + c;
+            if (valid && col < p.n_rows) p.logits[(size_t)(p.row0 + col) * p.V + vid] = x[c];
+          }
+        }
 #pragma unroll
         for (int c = 0; c < 16; ++c) {
           const int col = ch * 16 + c;   // < n_mma; s_draft holds -2 past n_rows
@@ -583,7 +571,7 @@ bool make_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, 
 }  // namespace
 
 // Limits already set on each variant of the kernel.
-template <bool KEYED>
+template <int MODE>
 KernelLimits& lm_limits() {
   static KernelLimits lim;
   return lim;
@@ -615,16 +603,24 @@ LmheadPlan plan_lmhead(int M, int d, int V, int num_sms) {
 cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
                           const __nv_bfloat16* w, const int32_t* draft_for_row, int32_t* argmax,
                           float* stats, void* ws, const LmheadPlan& pl, int* err,
-                          cudaStream_t stream, const unsigned long long* seed, float inv_temp) {
+                          cudaStream_t stream, const unsigned long long* seed, float inv_temp,
+                          float* logits) {
   const bool keyed = seed != nullptr;
+  const int mode = keyed ? MODE_KEYED : logits ? MODE_LOGITS : MODE_GREEDY;
   CUtensorMap map_w, map_h;
   if (!make_map(&map_w, w, (uint64_t)V, (uint64_t)d, BM)) return cudaErrorInvalidValue;
   if (!make_map(&map_h, hidden, (uint64_t)M, (uint64_t)d, (uint32_t)pl.n_mma))
     return cudaErrorInvalidValue;
   {
     const cudaError_t e =
-        keyed ? ensure_kernel_limits((const void*)lmhead_kernel<true>, lm_limits<true>(), 227 * 1024, false)
-              : ensure_kernel_limits((const void*)lmhead_kernel<false>, lm_limits<false>(), 227 * 1024, false);
+        mode == MODE_KEYED
+            ? ensure_kernel_limits((const void*)lmhead_kernel<MODE_KEYED>, lm_limits<MODE_KEYED>(),
+                                   227 * 1024, false)
+        : mode == MODE_LOGITS
+            ? ensure_kernel_limits((const void*)lmhead_kernel<MODE_LOGITS>,
+                                   lm_limits<MODE_LOGITS>(), 227 * 1024, false)
+            : ensure_kernel_limits((const void*)lmhead_kernel<MODE_GREEDY>,
+                                   lm_limits<MODE_GREEDY>(), 227 * 1024, false);
     if (e != cudaSuccess) return e;
   }
   float4* part = static_cast<float4*>(ws);
@@ -641,6 +637,7 @@ cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
     p.part_k = part_k;
     p.seed = seed;
     p.inv_temp = inv_temp;
+    p.logits = logits;
     p.row0 = pass * MAX_ROWS;
     p.n_rows = (M - p.row0) < MAX_ROWS ? (M - p.row0) : MAX_ROWS;
     p.n_mma = pl.n_mma;
@@ -653,15 +650,18 @@ cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
     const dim3 rgrid((p.n_rows + 3) / 4);
     cudaError_t e;
     if (keyed) {
-      e = launch_pdl(lmhead_kernel<true>, dim3(pl.grid), dim3(NUM_THREADS), pl.smem_bytes, stream,
-                     map_w, map_h, p);
+      e = launch_pdl(lmhead_kernel<MODE_KEYED>, dim3(pl.grid), dim3(NUM_THREADS), pl.smem_bytes,
+                     stream, map_w, map_h, p);
       if (e != cudaSuccess) return e;
       e = launch_pdl(lmhead_reduce_kernel<true>, rgrid, dim3(128), 0, stream, (const float4*)part,
                      (const int*)part_idx, (const float*)part_k, pl.grid, p.row0, p.n_rows, V,
                      draft_for_row, argmax, stats, err);
     } else {
-      e = launch_pdl(lmhead_kernel<false>, dim3(pl.grid), dim3(NUM_THREADS), pl.smem_bytes, stream,
-                     map_w, map_h, p);
+      e = mode == MODE_LOGITS
+              ? launch_pdl(lmhead_kernel<MODE_LOGITS>, dim3(pl.grid), dim3(NUM_THREADS),
+                           pl.smem_bytes, stream, map_w, map_h, p)
+              : launch_pdl(lmhead_kernel<MODE_GREEDY>, dim3(pl.grid), dim3(NUM_THREADS),
+                           pl.smem_bytes, stream, map_w, map_h, p);
       if (e != cudaSuccess) return e;
       e = launch_pdl(lmhead_reduce_kernel<false>, rgrid, dim3(128), 0, stream, (const float4*)part,
                      (const int*)part_idx, (const float*)nullptr, pl.grid, p.row0, p.n_rows, V,
@@ -745,7 +745,8 @@ extern "C" COSPEC_API int cospec_lmhead_argmax_features_noalloc(
       !make_map(&map_h, hidden, (uint64_t)M, (uint64_t)d, (uint32_t)pl.n_mma))
     return cuda_status(cudaErrorInvalidValue);      // as the workspace entry point reports it
   const cudaError_t le =
-      ensure_kernel_limits((const void*)lmhead_kernel<false>, lm_limits<false>(), 227 * 1024, false);
+      ensure_kernel_limits((const void*)lmhead_kernel<MODE_GREEDY>, lm_limits<MODE_GREEDY>(),
+                           227 * 1024, false);
   if (le != cudaSuccess) return cuda_status(le);
   uint32_t tmem_cols = 32;
   while (tmem_cols < (uint32_t)(2 * pl.n_mma)) tmem_cols <<= 1;
@@ -766,7 +767,7 @@ extern "C" COSPEC_API int cospec_lmhead_argmax_features_noalloc(
     p.stages = pl.stages;
     p.tmem_cols = tmem_cols;
     p.err = err;
-    cudaError_t e = launch_pdl(lmhead_kernel<false>, dim3(pl.grid), dim3(NUM_THREADS),
+    cudaError_t e = launch_pdl(lmhead_kernel<MODE_GREEDY>, dim3(pl.grid), dim3(NUM_THREADS),
                                pl.smem_bytes, st, map_w, map_h, p);
     if (e == cudaSuccess)
       e = launch_pdl(lmhead_reduce_kernel<false>, dim3((p.n_rows + 3) / 4), dim3(128), 0, st,

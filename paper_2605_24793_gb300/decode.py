@@ -2,7 +2,11 @@
 draft, verify, arbitrate, stop at the first rejected mismatch, commit,
 repeat) and the mean accepted length tau = (1/R) sum_r s^(r) (Sec. 3.1, Eq. 5).
 With a temperature, target candidates are drawn by sampling (stochastic
-decoding, Sec. 3.1) with a fresh seed per round from a device table.
+decoding, Sec. 3.1) with a fresh seed per round from a device table.  With
+``sps`` the rounds are those of the exact-match baseline with speculative
+sampling at that temperature (the paper's distribution-preserving comparison
+at T = 1): each round's drafts are drawn from a synthetic draft distribution
+(the target's logits plus Gaussian noise), kept in a device table with them.
 
 The rounds reuse one CUDA graph: every replay copies that round's draft ids
 from a device table (selected by a device-side round counter), runs the
@@ -14,6 +18,7 @@ block (Q, block K/V, hidden rows) are the workload's synthetic tensors.
   python -m paper_2605_24793_gb300.decode --config qwen3_8b_b1 --rounds 64
   python -m paper_2605_24793_gb300.decode --sweep        # K and lambda sweep
   python -m paper_2605_24793_gb300.decode --temperature 1
+  python -m paper_2605_24793_gb300.decode --temperature 1 --sps   # the baseline
 """
 from __future__ import annotations
 
@@ -29,6 +34,14 @@ from . import workload as W
 from .round import VerifyRound
 
 
+def target_logits(cfg: W.RoundConfig, hidden: torch.Tensor, w: torch.Tensor) -> np.ndarray:
+    """fp32 logits of the block rows on the device, [B, R, V] on the host, used
+    only to synthesise draft distributions."""
+    h = hidden.float()
+    out = [(h[r0:r0 + 64] @ w.float().T).cpu() for r0 in range(0, h.shape[0], 64)]
+    return torch.cat(out).numpy().reshape(cfg.batch, cfg.rows, -1)
+
+
 def target_ranked_ids(cfg: W.RoundConfig, hidden: torch.Tensor, w: torch.Tensor, t: int = 8):
     """Ranked top-t ids of each block row's logits (fp32 on the device), used
     only to synthesise draft ids."""
@@ -42,21 +55,34 @@ def target_ranked_ids(cfg: W.RoundConfig, hidden: torch.Tensor, w: torch.Tensor,
 class MultiRoundDecoder:
     def __init__(self, cfg: W.RoundConfig, rounds: int, lam: Optional[float] = None,
                  mode: int = C.POLICY_MLP, device="cuda", inputs: Optional[Dict] = None,
-                 drafts: Optional[np.ndarray] = None, temperature: Optional[float] = None):
+                 drafts: Optional[np.ndarray] = None, temperature: Optional[float] = None,
+                 sps: bool = False, draft_noise: float = 1.0):
         self.cfg, self.rounds = cfg, rounds
         self.lam = cfg.lam if lam is None else lam
         self.inp = inputs if inputs is not None else W.make_round_inputs(
             cfg, device=device, extra_tokens=rounds * cfg.rows)
+        dev = self.inp["q"].device
+        self.sps = sps
+        self.q_table = None
+        if sps:
+            if temperature is None:
+                temperature = 1.0
+            x = target_logits(cfg, self.inp["hidden"], self.inp["w"])
+            qs = [W.draft_distributions(cfg, x, draft_noise, temperature, r) for r in range(rounds)]
+            if drafts is None:
+                drafts = np.stack([W.sample_from(cfg, q, r) for r, q in enumerate(qs)])
+            self.q_table = torch.from_numpy(np.stack(qs)).to(dev)
+            del x, qs
         if drafts is None:
             ranked = target_ranked_ids(cfg, self.inp["hidden"], self.inp["w"])
             drafts = np.stack([W.synth_drafts(cfg, ranked, r) for r in range(rounds)])
         self.drafts_np = drafts
-        dev = self.inp["q"].device
         max_ctx = int(self.inp["ctx_len_np"].max()) + rounds * cfg.rows
         self.temperature = temperature
         self.seeds_np = np.array([W.sample_seed(cfg, r) for r in range(rounds)], dtype=np.int64)
         self.rnd = VerifyRound(self.inp, drafts[0], self.lam, mode, max_ctx=max_ctx,
-                               temperature=temperature, seed=int(self.seeds_np[0]))
+                               temperature=temperature, seed=int(self.seeds_np[0]),
+                               sps_q=None if self.q_table is None else self.q_table[0].clone())
         B, K, R = cfg.batch, cfg.k, cfg.rows
         dfr = np.full((rounds, B, R), -1, dtype=np.int32)
         dfr[:, :, :K] = drafts
@@ -74,6 +100,9 @@ class MultiRoundDecoder:
         torch.index_select(self.dfr, 0, self.idx, out=self.rnd.draft_for_row.view(1, -1))
         if self.temperature is not None:
             torch.index_select(self.seeds, 0, self.idx, out=self.rnd.seed)
+        if self.q_table is not None:
+            torch.index_select(self.q_table, 0, self.idx,
+                               out=self.rnd.draft_q.view((1,) + tuple(self.rnd.draft_q.shape)))
         self.rnd.run(restore=False)
         self.s_hist.index_copy_(0, self.idx, self.rnd.accept_len.view(1, B))
         self.emitted_hist.index_copy_(0, self.idx, self.rnd.emitted.view(1, B, -1))
@@ -129,6 +158,10 @@ def main():
     ap.add_argument("--lam", type=float, default=None)
     ap.add_argument("--temperature", type=float, default=None,
                     help="sample target candidates at this temperature (default: greedy)")
+    ap.add_argument("--sps", action="store_true",
+                    help="the exact-match baseline with speculative sampling (T = 1 by default)")
+    ap.add_argument("--draft-noise", type=float, default=1.0,
+                    help="std of the noise added to the target logits to form the draft (--sps)")
     ap.add_argument("--sweep", action="store_true",
                     help="K in {15, 20, 25} at lambda 0.6, then lambda in {0.4, 0.6, 0.8} at K 25")
     args = ap.parse_args()
@@ -142,10 +175,13 @@ def main():
         points = [(args.k if args.k is not None else base.k, args.lam if args.lam is not None else base.lam)]
     for k, lam in points:
         cfg = base.replace(k=k)
-        dec = MultiRoundDecoder(cfg, args.rounds, lam, temperature=args.temperature)
+        dec = MultiRoundDecoder(cfg, args.rounds, lam, temperature=args.temperature, sps=args.sps,
+                                draft_noise=args.draft_noise)
         res = dec.run()
         res.update({"workload": cfg.name, "k": k, "lambda": lam, "batch": cfg.batch,
-                    "temperature": args.temperature})
+                    "temperature": dec.temperature,
+                    "method": "exact-match, speculative sampling" if args.sps else "CoSpec",
+                    "draft_noise": args.draft_noise if args.sps else None})
         print(json.dumps(res), flush=True)
         del dec
         torch.cuda.empty_cache()

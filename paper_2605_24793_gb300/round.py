@@ -20,11 +20,18 @@ from . import cospec as C
 class VerifyRound:
     def __init__(self, inputs: Dict[str, object], draft: np.ndarray, lam: float = 0.6,
                  mode: int = C.POLICY_MLP, keep_attn: bool = False, max_ctx: Optional[int] = None,
-                 temperature: Optional[float] = None, seed: int = 0):
+                 temperature: Optional[float] = None, seed: int = 0,
+                 sps_q: Optional[torch.Tensor] = None):
         """``temperature`` None: greedy target candidates (argmax).  Otherwise
         stochastic decoding (Sec. 3.1): candidates are Gumbel-max samples at
         that temperature, keyed by the device scalar ``self.seed``, which a
-        caller may rewrite between replays of a captured round."""
+        caller may rewrite between replays of a captured round.
+
+        ``sps_q`` [B, K, V] fp32 (the draft's distributions) turns the round
+        into the exact-match baseline with speculative sampling at
+        ``temperature`` (1 when None): the LM head writes the scaled logits,
+        the acceptance step replaces arbitration, and the commit takes its
+        tokens."""
         cfg = inputs["cfg"]
         self.cfg = cfg
         self.inp = inputs
@@ -57,6 +64,17 @@ class VerifyRound:
         self.emitted = torch.empty((B, R), dtype=torch.int32, device=dev)
         self.temperature = None if temperature is None else float(temperature)
         self.seed = torch.tensor([int(seed)], dtype=torch.int64, device=dev)
+        self.sps = sps_q is not None
+        if self.sps:
+            if self.temperature is None:
+                self.temperature = 1.0
+            if tuple(sps_q.shape) != (B, K, cfg.vocab):
+                raise ValueError("sps_q must be [B, K, V]")
+            self.draft_q = sps_q
+            self.logits = torch.empty((M, cfg.vocab), dtype=torch.float32, device=dev)
+            self.target = torch.empty(M, dtype=torch.int32, device=dev)
+            self.ratio = torch.empty((B, K), dtype=torch.float32, device=dev)
+            self.ws_sps = C.new_sps_workspace(B, dev)
         self.graph: Optional[torch.cuda.CUDAGraph] = None
         self.launches_per_round = self._count_launches()
 
@@ -93,7 +111,8 @@ class VerifyRound:
         accept/commit: commit + scan)."""
         cfg = self.cfg
         passes = (cfg.m_rows + 255) // 256
-        return cfg.layers + 2 * passes + (1 if cfg.k > 0 else 0) + 2
+        decide = 2 if self.sps else (1 if cfg.k > 0 else 0)
+        return cfg.layers + 2 * passes + decide + 2
 
     def restore_context(self) -> None:
         """Reset ctx_len to the round's starting context (device copy)."""
@@ -111,6 +130,10 @@ class VerifyRound:
                              kv_stable=(l > 0) if kv_stable is None else kv_stable)
 
     def lmhead(self):
+        if self.sps:
+            return C.lmhead_logits_features(self.hidden, self.w, self.draft_for_row,
+                                            self.temperature, self.argmax, self.stats,
+                                            self.logits, self.ws_lm)
         if self.temperature is not None:
             return C.lmhead_sample_features(self.hidden, self.w, self.draft_for_row,
                                             self.temperature, self.seed, self.argmax, self.stats,
@@ -120,12 +143,16 @@ class VerifyRound:
 
     def arbitrate(self):
         cfg = self.cfg
+        if self.sps:
+            return C.sps_accept(self.draft, self.stats, self.logits, self.draft_q, self.seed,
+                                self.target, self.accept, self.ratio, self.ws_sps)
         return C.arbitrate(self.draft, self.argmax.view(cfg.batch, cfg.rows),
                            self.stats.view(cfg.batch, cfg.rows, 5), self.w1, self.b1, self.w2,
                            self.b2, self.lam, self.mode, self.p, self.accept)
 
     def commit(self):
-        return C.accept_commit(self.draft, self.argmax, self.accept, self.k_blk, self.v_blk,
+        tokens = self.target if self.sps else self.argmax
+        return C.accept_commit(self.draft, tokens, self.accept, self.k_blk, self.v_blk,
                                self.k_pages, self.v_pages, self.page_table, self.ctx_len,
                                self.accept_len, self.emitted)
 
@@ -136,7 +163,7 @@ class VerifyRound:
         for l in range(self.cfg.layers):
             self.attention(l)
         self.lmhead()
-        if self.cfg.k > 0:
+        if self.cfg.k > 0 or self.sps:
             self.arbitrate()
         self.commit()
 

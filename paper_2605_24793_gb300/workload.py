@@ -307,15 +307,16 @@ def rl_batch(seed: int, groups: int, rollouts: int, rounds: int, k: int,
 
 
 def draft_distributions(cfg: RoundConfig, logits: np.ndarray, noise: float = 1.0,
-                        temperature: float = 1.0) -> np.ndarray:
+                        temperature: float = 1.0, round_index: int = 0) -> np.ndarray:
     """A stand-in for the draft model's distributions at the K draft
     positions, for speculative sampling: q_i = softmax((x_{i-1} + noise * eps)
     / T) with eps ~ N(0, 1), where ``logits`` [B, R, V] are the target's
     logits of the block rows (whoever computed them) -- a draft that roughly
-    agrees with the target.  Returns float32 [B, K, V]."""
+    agrees with the target.  ``round_index`` selects an independent draw for
+    each round of a multi-round run.  Returns float32 [B, K, V]."""
     x = np.asarray(logits, dtype=np.float64)
     B, R, V = x.shape
-    rng = np.random.default_rng(seed_of(cfg, "draft_q"))
+    rng = np.random.default_rng(seed_of(cfg, "draft_q") + 7919 * round_index)
     z = (x[:, : R - 1] + noise * rng.standard_normal((B, R - 1, V))) / temperature
     z -= z.max(axis=-1, keepdims=True)
     e = np.exp(z)

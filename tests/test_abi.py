@@ -228,6 +228,29 @@ def test_sample_host_validation(lib):
     assert f(4, 4000, 1000, fake, fake, fake, 1.0, fake, fake, fake, fake, 1 << 30, None) == -2
 
 
+def test_logits_and_sps_host_validation(lib):
+    fake = ctypes.c_void_p(1 << 20)                                   # never dereferenced
+    f = lib.cospec_lmhead_logits_features
+    args = lambda T, logits: (4, 4096, 1000, fake, fake, fake, T, fake, fake, logits, fake, 1 << 30,
+                              None)
+    assert f(*args(0.0, fake)) == -1                                  # temperature must be > 0
+    assert f(*args(float("inf"), fake)) == -1
+    assert f(*args(1.0, None)) == -1                                  # logits pointer missing
+    assert f(*args(1.0, ctypes.c_void_p((1 << 20) + 2))) == -1        # logits not 4-byte aligned
+    assert f(0, 4096, 1000, *([None] * 3), 1.0, *([None] * 4), 0, None) == 0
+    g = lib.cospec_sps_accept
+    ws = lib.cospec_sps_workspace(8)
+    assert ws >= 8 * 64 * 16 and lib.cospec_sps_workspace(0) == 0
+    sargs = lambda B, K, seed, wsb: (B, K, 1000, fake, fake, fake, fake, seed, fake, fake, fake,
+                                     fake, wsb, None)
+    assert g(*sargs(8, 32, fake, ws)) == -2                           # K <= 31
+    assert g(*sargs(8, 5, None, ws)) == -1                            # seed missing
+    assert g(*sargs(8, 5, ctypes.c_void_p((1 << 20) + 4), ws)) == -1  # seed not 8-byte aligned
+    assert g(*sargs(8, 5, fake, ws - 1)) == -3                        # workspace too small
+    assert g(0, 5, 1000, *([None] * 9), 0, None) == 0                 # empty batch
+    assert g(8, 5, 1000, fake, fake, fake, None, fake, fake, fake, fake, fake, ws, None) == -1
+
+
 C_PROGRAM = r"""
 #include <stdio.h>
 #include <string.h>
