@@ -69,9 +69,11 @@ def attention_flops(cfg, ctx: np.ndarray) -> float:
     return 4.0 * cfg.rows * cfg.q_heads * cfg.head_dim * float(np.sum(ctx + cfg.rows))
 
 
-def lmhead_bytes(cfg) -> float:
-    """W streamed once plus the hidden rows and the per-row outputs."""
-    return 2.0 * cfg.vocab * cfg.hidden + 2.0 * cfg.m_rows * cfg.hidden + 24.0 * cfg.m_rows
+def lmhead_bytes(cfg, logits: bool = False) -> float:
+    """W streamed once plus the hidden rows and the per-row outputs (and the
+    M x V fp32 logits when the LM head writes them, speculative sampling)."""
+    b = 2.0 * cfg.vocab * cfg.hidden + 2.0 * cfg.m_rows * cfg.hidden + 24.0 * cfg.m_rows
+    return b + (4.0 * cfg.m_rows * cfg.vocab if logits else 0.0)
 
 
 def lmhead_flops(cfg) -> float:
@@ -320,13 +322,25 @@ def measure(cfg, args, env, inp=None, with_cpu=True, with_e2e=True):
     world, rank, local_rank, dist = env
     if inp is None:
         inp = W.make_round_inputs(cfg, device="cuda")
-    draft = gpu_drafts(cfg, inp)
+    sps_q = None
+    if args.sps:
+        # the exact-match baseline with speculative sampling: drafts drawn from
+        # a synthetic draft distribution (the target's logits plus noise)
+        from paper_2605_24793_gb300.decode import target_logits
+        q = W.draft_distributions(cfg, target_logits(cfg, inp["hidden"], inp["w"]),
+                                  args.draft_noise, args.temperature or 1.0)
+        draft = W.sample_from(cfg, q)
+        sps_q = torch.from_numpy(q).cuda()
+        del q
+    else:
+        draft = gpu_drafts(cfg, inp)
     rnd = VerifyRound(inp, draft, cfg.lam, temperature=args.temperature,
-                      seed=W.sample_seed(cfg))
+                      seed=W.sample_seed(cfg), sps_q=sps_q)
     rnd.pack_step_io()                    # one host->device and one device->host copy per step
     attn_kernel, attn_splits = C.verify_attn_plan(inp["q"][0], inp["k_pages"][0], inp["page_table"],
                                                   rnd.max_ctx)
-    lm_name = "lmhead_argmax_features" if args.temperature is None else "lmhead_sample_features"
+    lm_name = ("lmhead_logits_features" if args.sps else
+               "lmhead_argmax_features" if args.temperature is None else "lmhead_sample_features")
     stream = torch.cuda.Stream()
     torch.cuda.synchronize()
 
@@ -348,7 +362,7 @@ def measure(cfg, args, env, inp=None, with_cpu=True, with_e2e=True):
     g_lm = cap(rnd.lmhead)
 
     def tail():
-        if cfg.k > 0:
+        if cfg.k > 0 or rnd.sps:
             rnd.arbitrate()
         rnd.commit()
     g_tail = cap(tail)
@@ -446,7 +460,7 @@ def measure(cfg, args, env, inp=None, with_cpu=True, with_e2e=True):
     pk, pk_kind = peaks()
     ctx = inp["ctx_len_np"]
     a_bytes = attention_bytes(cfg, ctx)
-    lm_bytes = lmhead_bytes(cfg)
+    lm_bytes = lmhead_bytes(cfg, logits=rnd.sps)
     attn_launch_ms = attn_ms / cfg.layers
     hbm = float(pk["hbm_gbs"])
     tflops_peak = float(pk.get("bf16_tflops_sustained", pk["bf16_tflops"]))
@@ -477,7 +491,8 @@ def measure(cfg, args, env, inp=None, with_cpu=True, with_e2e=True):
                   "bound": "hbm" if lm_t_hbm >= lm_t_tc else "tensor",
                   "frac_roofline": max(lm_t_hbm, lm_t_tc) / (lm_ms * 1e-3),
                   "share": lm_ms / seg},
-        "arbitrate+accept_commit": {"ms_per_step": tail_ms, "share": tail_ms / seg},
+        ("sps_accept+accept_commit" if rnd.sps else "arbitrate+accept_commit"):
+            {"ms_per_step": tail_ms, "share": tail_ms / seg},
     }
     if attn_ms >= lm_ms:
         dom = "verify_attn"
@@ -529,7 +544,9 @@ def measure(cfg, args, env, inp=None, with_cpu=True, with_e2e=True):
                    "head_dim": cfg.head_dim, "hidden": cfg.hidden, "vocab": cfg.vocab,
                    "page_size": cfg.page_size, "lambda": cfg.lam,
                    "mismatch_rate": cfg.mismatch_rate,
-                   "decoding": ("greedy" if args.temperature is None
+                   "decoding": (f"exact-match speculative sampling, T={rnd.temperature}, draft "
+                                f"= target logits + N(0, {args.draft_noise}^2)" if rnd.sps else
+                                "greedy" if args.temperature is None
                                 else f"sampled, T={args.temperature}"),
                    "parallelism": f"replicas x{world}",
                    "l2": (f"inputs larger than L2: {(a_bytes * cfg.layers + lm_bytes) / 1e9:.2f}"
@@ -613,6 +630,11 @@ def main():
                     help="override the draft length K (block rows K+1), e.g. 25 as in the paper")
     ap.add_argument("--temperature", type=float, default=None,
                     help="stochastic decoding: sample the target candidates at this temperature")
+    ap.add_argument("--sps", action="store_true",
+                    help="time the exact-match baseline with speculative sampling (T = 1 unless "
+                         "--temperature) instead of the CoSpec round")
+    ap.add_argument("--draft-noise", type=float, default=1.0,
+                    help="--sps: std of the noise added to the target logits to form the draft")
     ap.add_argument("--sweep", action="store_true",
                     help="the Llama-3-8B batch-64 points (K x mismatch rate), one line each")
     ap.add_argument("--points", nargs="+", default=None, help="subset of the sweep's workloads")

@@ -80,13 +80,16 @@ class VerifyRound:
 
     def pack_step_io(self) -> None:
         """Place the inputs a serving step receives from the host (Q and the
-        block K/V of every layer, the hidden rows, the draft ids) in one device
+        block K/V of every layer, the hidden rows, the draft ids and, for
+        speculative sampling, the draft's distributions) in one device
         buffer ``io_in`` and the results it hands back (accepted lengths,
         emitted tokens) in another, ``io_out``, so that a step moves each with
         a single copy.  The tensors become views of the buffers (each slice
         256-byte aligned); call before capturing a graph."""
         dev = self.q.device
         names = ("q", "k_blk", "v_blk", "hidden", "draft", "draft_for_row")
+        if self.sps:
+            names += ("draft_q",)            # the draft's distributions come with the drafts
         tensors = [getattr(self, n) for n in names]
         sizes = [t.numel() * t.element_size() for t in tensors]
         offs, total = [], 0
