@@ -179,6 +179,10 @@ CS_DEV uint32_t cluster_nctarank() {
 // Cluster barrier in two halves, for work in between (every thread of the
 // CTA executes both, arrive first).
 CS_DEV void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
+// An arrival that orders no memory: for barriers that only say "this CTA is
+// past a point" (its ring is idle, or every copy addressed to it has landed),
+// where nothing written before the arrival is read through the barrier.
+CS_DEV void cluster_arrive_relaxed() { asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory"); }
 CS_DEV void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
 // Address of the same shared-memory location in CTA `rank` of the cluster.
 CS_DEV uint32_t dsmem_map(uint32_t local, uint32_t rank) {

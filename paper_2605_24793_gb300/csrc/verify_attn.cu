@@ -456,7 +456,7 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 64,
   const int rpo = (NR + S - 1) / S;      // rows finished by each owner
   if (S > 1) {
     if (tid == 0) mbar_arrive_expect_tx(recv_bar, (uint32_t)(S * rpo * LY::ROWP));
-    cluster_arrive();
+    cluster_arrive_relaxed();
   }
 
   // CTA partial: rows of every warp, key groups merged (stage ring reused).
@@ -550,7 +550,7 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 64,
     // Everything addressed to this CTA has landed.  Once every CTA has said
     // so, no copy reads or writes this CTA's shared memory any more: arrive
     // now, wait at the very end, and merge in between.
-    cluster_arrive();
+    cluster_arrive_relaxed();
   }
   const int row0 = rank * rpo;
   // Per owned row: one warp forms the common maximum over the S partials and

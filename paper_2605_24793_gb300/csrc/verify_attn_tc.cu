@@ -668,7 +668,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   const int rpo = (NR + S - 1) / S;      // rows finished by each owner
   if (S > 1) {
     if (tid == 0) mbar_arrive_expect_tx(recv_bar, (uint32_t)(S * rpo * LY::ROWP));
-    cluster_arrive();
+    cluster_arrive_relaxed();
   }
   float* part = reinterpret_cast<float*>(smem + LY::PART);
   const bool have = T > 0 && !*abort_flag;
@@ -720,7 +720,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
     if (!mbar_wait(recv_bar, 0)) set_err(p.err, ERR_TIMEOUT);
     src = recv;
-    cluster_arrive();                    // everything addressed to this CTA has landed
+    cluster_arrive_relaxed();            // everything addressed to this CTA has landed
   }
   const int row0 = rank * rpo;
   // Per owned row: one warp forms the common maximum over the S partials and
