@@ -151,10 +151,13 @@ typedef struct {
  * for one round. */
 #define COSPEC_ATTN_BLOCK_FULL 2
 
-/* Launch plan cospec_verify_attn would use for these dimensions on the
- * current device: *kernel = 0 (mma.sync) or 1 (tcgen05), *splits = CTAs per
- * (sequence, KV head, row group).  Host only; returns COSPEC_OK or the error
- * cospec_verify_attn would return for the dimensions. */
+/* Launch plan cospec_verify_attn would use for these dimensions (flags
+ * included: a small batch launched with COSPEC_ATTN_KV_STABLE, which may
+ * overlap the kernel before it, can take a larger KV split than one that
+ * starts on an idle GPU) on the current device: *kernel = 0 (mma.sync) or 1
+ * (tcgen05), *splits = CTAs per (sequence, KV head, row group), 1 to 16.
+ * Host only; returns COSPEC_OK or the error cospec_verify_attn would return
+ * for the dimensions. */
 COSPEC_API int cospec_verify_attn_plan(const cospec_attn_dims* dims, int max_ctx, int* kernel,
                                        int* splits);
 

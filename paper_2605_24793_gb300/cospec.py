@@ -218,9 +218,10 @@ def num_sms() -> int:
 ATTN_MMA_SYNC, ATTN_TCGEN05 = 0, 1
 
 
-def verify_attn_plan(q, k_pages, page_table, max_ctx: int):
-    """(kernel, splits) cospec_verify_attn would use for these tensors."""
-    dims = attn_dims(q, k_pages, page_table)
+def verify_attn_plan(q, k_pages, page_table, max_ctx: int, kv_stable: bool = False):
+    """(kernel, splits) cospec_verify_attn would use for these tensors (and
+    the stable-cache flag, which the plan of small batches depends on)."""
+    dims = attn_dims(q, k_pages, page_table, flags=ATTN_KV_STABLE if kv_stable else 0)
     kernel, splits = ctypes.c_int(), ctypes.c_int()
     _check(load_library().cospec_verify_attn_plan(ctypes.byref(dims), int(max_ctx),
                                                   ctypes.byref(kernel), ctypes.byref(splits)))

@@ -91,7 +91,7 @@ struct AttnPlan {
 // device (0: not schedulable).
 using ResidentFn = std::function<long long(const AttnPlan&, int S)>;
 AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int num_sms,
-                          const ResidentFn& resident);
+                          bool kv_stable, const ResidentFn& resident);
 int attn_max_active_clusters(int D, int mt, int wk, int S, int Hkv, int B, int kbr);
 cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& plan, int* err,
                                cudaStream_t stream);

@@ -674,7 +674,7 @@ int variant_mt(int NR) {   // NR <= 64
 }  // namespace
 
 AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int num_sms,
-                          const ResidentFn& resident) {
+                          bool kv_stable, const ResidentFn& resident) {
   AttnPlan pl{};
   const int NRT = (Hq / Hkv) * R;
   const int RG = (NRT + 63) / 64;                  // row groups of at most 64 rows
@@ -713,7 +713,17 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
     // a small batch (latency-bound): every cluster resident at once, and
     // down to two tiles per CTA
     pl.one_wave = (pl.units * 4 <= num_sms && len_tc <= 1) ? 1 : 0;
-    const int min_tiles = pl.one_wave ? 2 : 8;
+    if (pl.one_wave) {
+      // the largest split of any size up to 16 whose clusters are all resident
+      // at once (batch 1, K = 15: 12 splits 11.6 us per layer against 12.5 with 8
+      // and 19.7 with 16, a second wave; K = 25, two row groups: 16.5 us with 4
+      // splits, 23.7 with 8, whose 16 clusters do not fit at once)
+      int s = 16;
+      while (s > 1 && (s * 2 > tiles_tc || resident(pl, s) < pl.units)) --s;
+      pl.cluster = s;
+      return pl;
+    }
+    const int min_tiles = 8;
     while (S < 16 && S < want_tc && (S * 2) * min_tiles <= tiles_tc) S *= 2;
   } else {
     // Split each (sequence, head, row group) over a cluster of S CTAs: about
@@ -732,16 +742,25 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
     // A batch of a few units (at most a quarter of the slots) is bound by the
     // latency of one CTA's tile loop and the cluster merge, and a second wave
     // of clusters (the GPU places whole clusters inside one GPC) doubles it:
-    // take the largest split whose clusters are all resident at once.
+    // take the largest even split up to 16, at least four tiles per CTA,
+    // whose clusters are all resident at once (Qwen3-8B batch 2: 12 splits
+    // 10.7 us per layer, 8 12.5 us, 16 -- a second wave -- 16.2 us; at two
+    // CTAs per SM an odd cluster leaves an SM shared with another cluster:
+    // 13 splits 11.9 us).
+    // A launch that may not overlap the kernel before it (no stable-cache
+    // promise) starts on an idle GPU, where at batch 1 12 splits ran 8.2-8.9 us
+    // against 10.3-10.9 us with 16; back to back, 16 stays faster (8.8 against
+    // 9.8 us with 12).
     pl.one_wave = (pl.units * 4 <= slots && want_len <= 1) ? 1 : 0;
+    if (pl.one_wave) {
+      int s = kv_stable ? 16 : 12;
+      while (s > 1 && (s * 4 > tiles || resident(pl, s) < pl.units)) s = s > 2 ? s - 2 : 1;
+      pl.cluster = s;
+      return pl;
+    }
   }
-  // the largest cluster not above S that can be scheduled at all (and, for a
-  // one-wave launch, with every cluster resident)
-  while (S > 1) {
-    const long long n = resident(pl, S);
-    if (n > 0 && (!pl.one_wave || n >= pl.units)) break;
-    S >>= 1;
-  }
+  // the largest cluster not above S that can be scheduled at all
+  while (S > 1 && resident(pl, S) <= 0) S >>= 1;
   pl.cluster = S;
   return pl;
 }

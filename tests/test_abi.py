@@ -87,11 +87,13 @@ def test_attention_plan_host_validation(lib):
 
 
 # Clusters of S CTAs resident at once on a GB300 (152 SMs), from
-# cudaOccupancyMaxActiveClusters for every attention variant: two CTAs per SM
-# for the mma.sync kernel with <= 32 block keys, one otherwise (and for the
-# tcgen05 kernel).
-_GB300_TWO_PER_SM = {1: 304, 2: 152, 4: 74, 8: 36, 16: 14}
-_GB300_ONE_PER_SM = {1: 152, 2: 76, 4: 36, 8: 15, 16: 7}
+# cudaOccupancyMaxActiveClusters for every attention variant and S = 1..16:
+# two CTAs per SM for the mma.sync kernel with <= 32 block keys, one otherwise
+# (and for the tcgen05 kernel).
+_GB300_TWO_PER_SM = dict(enumerate([304, 152, 97, 74, 58, 46, 38, 36, 30, 28, 23, 23, 19, 14, 14,
+                                    14], start=1))
+_GB300_ONE_PER_SM = dict(enumerate([152, 76, 46, 36, 28, 23, 15, 15, 15, 13, 8, 8, 7, 7, 7, 7],
+                                   start=1))
 
 
 def _gb300_resident(kernel, rows, block_rows, splits):
@@ -99,34 +101,45 @@ def _gb300_resident(kernel, rows, block_rows, splits):
     return table.get(splits, 0)
 
 
-# (batch, rows, Hq, Hkv, head_dim, longest context) -> (kernel, splits): the
-# planner's choice for each workload shape, which is also the fastest of the
-# splits timed on a GB300 (Qwen3-8B batch 16: 4 splits against 2 and 8;
-# Llama-3-8B batch 64: 2 against 4 and 8; Qwen3-32B batch 32: unsplit
-# against 2; Qwen3-8B batch 16 K = 15: 2 against 4).
+# (batch, rows, Hq, Hkv, head_dim, longest context, stable-cache flag) ->
+# (kernel, splits): the planner's choice for each workload shape, which is
+# also the fastest of the splits timed on a GB300 (Qwen3-8B batch 16: 4 splits
+# against 2 and 8; Llama-3-8B batch 64: 2 against 4 and 8; Qwen3-32B batch
+# 32: unsplit against 2; Qwen3-8B batch 16 K = 15: 2 against 4; batch 1, K = 5:
+# 16 back to back, 12 alone; batch 2: 12 against 13, 8 and 16; batch 4: 8
+# against 12 and 16; batch 1, K = 15: 12 against 8 and 16; K = 25: 6 against
+# 4 and 8).
 PLAN_CASES = [
-    ((1, 6, 32, 8, 128, 4096), (C.ATTN_MMA_SYNC, 16)),      # Qwen3-8B, batch 1, K = 5
-    ((16, 8, 32, 8, 128, 8192), (C.ATTN_MMA_SYNC, 4)),      # Qwen3-8B, batch 16, K = 7
-    ((1, 16, 32, 8, 128, 4096), (C.ATTN_TCGEN05, 8)),       # batch 1, K = 15: one wave
-    ((16, 16, 32, 8, 128, 8192), (C.ATTN_TCGEN05, 2)),      # batch 16, K = 15
-    ((32, 8, 64, 8, 128, 16384), (C.ATTN_TCGEN05, 1)),      # Qwen3-32B, batch 32
-    ((64, 8, 32, 8, 128, 32768), (C.ATTN_MMA_SYNC, 2)),     # Llama-3-8B, batch 64
+    ((1, 6, 32, 8, 128, 4096, 1), (C.ATTN_MMA_SYNC, 16)),   # Qwen3-8B, batch 1, K = 5
+    ((1, 6, 32, 8, 128, 4096, 0), (C.ATTN_MMA_SYNC, 12)),   # the same, on an idle GPU
+    ((2, 6, 32, 8, 128, 4096, 1), (C.ATTN_MMA_SYNC, 12)),   # batch 2: 16 clusters at once
+    ((4, 6, 32, 8, 128, 4096, 1), (C.ATTN_MMA_SYNC, 8)),    # batch 4: 32 clusters at once
+    ((16, 8, 32, 8, 128, 8192, 1), (C.ATTN_MMA_SYNC, 4)),   # Qwen3-8B, batch 16, K = 7
+    ((1, 16, 32, 8, 128, 4096, 1), (C.ATTN_TCGEN05, 12)),   # batch 1, K = 15: one wave
+    ((1, 26, 32, 8, 128, 4096, 1), (C.ATTN_TCGEN05, 6)),    # batch 1, K = 25: 16 clusters
+    ((16, 16, 32, 8, 128, 8192, 1), (C.ATTN_TCGEN05, 2)),   # batch 16, K = 15
+    ((32, 8, 64, 8, 128, 16384, 1), (C.ATTN_TCGEN05, 1)),   # Qwen3-32B, batch 32
+    ((64, 8, 32, 8, 128, 32768, 1), (C.ATTN_MMA_SYNC, 2)),  # Llama-3-8B, batch 64
 ]
 
 
 @pytest.mark.parametrize("shape,plan", PLAN_CASES, ids=lambda v: str(v))
 def test_attention_plan_on_a_gb300_model(lib, shape, plan):
-    B, R, Hq, Hkv, D, ctx = shape
-    dims = C.AttnDims(B, R, Hq, Hkv, D, 16, (ctx + R + 15) // 16, 1 << 20, 0.0, 0)
+    B, R, Hq, Hkv, D, ctx, stable = shape
+    dims = C.AttnDims(B, R, Hq, Hkv, D, 16, (ctx + R + 15) // 16, 1 << 20, 0.0,
+                      C.ATTN_KV_STABLE if stable else 0)
     assert C.verify_attn_plan_model(dims, ctx, 152, _gb300_resident) == plan
 
 
 def test_attention_plan_model_rules(lib):
-    # a batch of a few units: the largest split whose clusters are all resident
+    # a batch of a few units: the largest even split up to 16 whose clusters
+    # are all resident; at most 12 without the stable-cache promise
+    st = C.AttnDims(1, 6, 32, 8, 128, 16, 300, 1 << 20, 0.0, C.ATTN_KV_STABLE)
     dims = C.AttnDims(1, 6, 32, 8, 128, 16, 300, 1 << 20, 0.0, 0)
-    assert C.verify_attn_plan_model(dims, 4096, 152, lambda k, r, kb, s: 304 // s) == (0, 16)
-    assert C.verify_attn_plan_model(dims, 4096, 152, lambda k, r, kb, s: 7 if s >= 16 else 304 // s) \
-        == (0, 8)
+    assert C.verify_attn_plan_model(st, 4096, 152, lambda k, r, kb, s: 304 // s) == (0, 16)
+    assert C.verify_attn_plan_model(dims, 4096, 152, lambda k, r, kb, s: 304 // s) == (0, 12)
+    assert C.verify_attn_plan_model(st, 4096, 152, lambda k, r, kb, s: 7 if s >= 14 else 304 // s) \
+        == (0, 12)
     # no cluster of more than one CTA can be scheduled: no split
     assert C.verify_attn_plan_model(dims, 4096, 152, lambda k, r, kb, s: 152 if s == 1 else 0) \
         == (0, 1)

@@ -140,7 +140,7 @@ ATTN_TC_SPLIT_CASES = [
     # B, R, Hq, Hkv, D, contexts, shuffled, expected splits
     (12, 8, 64, 8, 128, [6000] + _ctx(11, 8), True, 2),           # 96 units
     (6, 8, 64, 8, 128, [9000, 3000] + _ctx(4, 9), True, 4),       # 48 units
-    (1, 8, 64, 8, 128, [6000], False, 8),                         # one wave of 8-CTA clusters
+    (1, 8, 64, 8, 128, [6000], False, 12),                        # one wave of 12-CTA clusters
     (20, 8, 64, 8, 128, [33000, 9000] + _ctx(18, 10), False, 2),  # a context past 256 tiles
 ]
 
@@ -366,10 +366,12 @@ def test_features_feed_the_mlp_as_the_oracle_builds_them():
         assert_close(z[mism], feats[..., k][mism], f"feature F{k}", abs_tol=1e-3, rel_tol=1e-3)
 
 
-@pytest.mark.parametrize("K", [0, 1, 5, 7])
-def test_accept_commit_matches_oracle(K):
-    rng = np.random.default_rng(40 + K)
-    L, B, R, Hkv, D, P = 3, 6, K + 1, 8, 128, 16
+@pytest.mark.parametrize("K,L,B", [(0, 3, 6), (1, 3, 6), (5, 3, 6), (7, 3, 6), (7, 64, 32)])
+def test_accept_commit_matches_oracle(K, L, B):
+    # (7, 64, 32): the commit grid of the Qwen3-32B-shaped round (64 layers x
+    # 32 sequences, one CTA each), with short contexts
+    rng = np.random.default_rng(40 + K + L)
+    R, Hkv, D, P = K + 1, 8, 128, 16
     ctx = rng.integers(0, 200, B).astype(np.int32)
     need = (ctx + R + P - 1) // P
     num = int(need.sum())
