@@ -579,10 +579,14 @@ KernelLimits& lm_limits() {
 
 LmheadPlan plan_lmhead(int M, int d, int V, int num_sms) {
   LmheadPlan pl{};
-  const int rows = M < MAX_ROWS ? M : MAX_ROWS;
+  // Rows beyond 256 take several passes over W, of equal size: a pass of
+  // 256 rows is tensor-bound while a short one is bound by streaming W, so
+  // 384 rows run as 2 x 192 rather than 256 + 128.  Pass p covers rows
+  // [p * n_mma, min(M, (p + 1) * n_mma)).
+  pl.passes = (M + MAX_ROWS - 1) / MAX_ROWS;
+  const int rows = (M + pl.passes - 1) / pl.passes;
   pl.n_mma = (rows + 15) / 16 * 16;
   if (pl.n_mma < 16) pl.n_mma = 16;
-  pl.passes = (M + MAX_ROWS - 1) / MAX_ROWS;
   pl.num_tiles = (V + BM - 1) / BM;
   pl.grid = pl.num_tiles < num_sms ? pl.num_tiles : num_sms;
   // One plan serves both variants: shared memory is sized for the keyed
@@ -638,8 +642,8 @@ cudaError_t launch_lmhead(int M, int d, int V, const __nv_bfloat16* hidden,
     p.seed = seed;
     p.inv_temp = inv_temp;
     p.logits = logits;
-    p.row0 = pass * MAX_ROWS;
-    p.n_rows = (M - p.row0) < MAX_ROWS ? (M - p.row0) : MAX_ROWS;
+    p.row0 = pass * pl.n_mma;
+    p.n_rows = (M - p.row0) < pl.n_mma ? (M - p.row0) : pl.n_mma;
     p.n_mma = pl.n_mma;
     p.d = d;
     p.V = V;
@@ -758,8 +762,8 @@ extern "C" COSPEC_API int cospec_lmhead_argmax_features_noalloc(
     p.stats = stats;
     p.part = part;
     p.part_idx = part_idx;
-    p.row0 = pass * MAX_ROWS;
-    p.n_rows = (M - p.row0) < MAX_ROWS ? (M - p.row0) : MAX_ROWS;
+    p.row0 = pass * pl.n_mma;
+    p.n_rows = (M - p.row0) < pl.n_mma ? (M - p.row0) : pl.n_mma;
     p.n_mma = pl.n_mma;
     p.d = d;
     p.V = V;

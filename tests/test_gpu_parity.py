@@ -267,8 +267,11 @@ LM_CASES = [
     (6, 4096, 151936, 0.02),      # Qwen3-8B LM head, batch 1, K = 5
     (17, 256, 1000, 0.1),         # vocabulary not a multiple of the 128-row tile
     (128, 1024, 3000, 0.05),
-    (300, 128, 2048, 0.1),        # two 256-row passes
+    (300, 128, 2048, 0.1),        # two passes of 160 and 140 rows
     (256, 5120, 1280, 0.02),
+    (384, 256, 3000, 0.05),       # two equal passes of 192 rows (the Llama K = 5 round)
+    (512, 256, 2000, 0.05),       # two full 256-row passes
+    (520, 128, 1500, 0.1),        # three passes of 176, 176 and 168 rows
 ]
 
 
@@ -544,7 +547,7 @@ SAMPLE_CASES = [
     (1, 64, 128, 0.1, 1.0, 0),
     (6, 4096, 151936, 0.02, 1.0, 0x0123456789ABCDEF),   # Qwen3-8B LM head, batch 1, K = 5
     (17, 256, 1000, 0.1, 0.5, 7),                      # ragged vocabulary tile, rows not 4-aligned
-    (300, 128, 2048, 0.1, 1.0, 2 ** 40 + 3),           # two 256-row passes
+    (300, 128, 2048, 0.1, 1.0, 2 ** 40 + 3),           # two passes (160 + 140 rows)
     (64, 512, 4096, 0.3, 2.0, 99),
 ]
 
