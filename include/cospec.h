@@ -117,9 +117,10 @@ COSPEC_API int cospec_num_sms(void);
  *    No workspace: the KV range of a (sequence, KV head) is split over the
  *    CTAs of one thread-block cluster, whose partial results merge in
  *    distributed shared memory.  Two kernels implement the call: one on
- *    mma.sync tensor-core tiles, and one on tcgen05 (TMEM accumulators),
- *    used when a row group of a KV head has more than 32 query rows (and at
- *    most 64 query heads share the KV head).  Sequences are processed
+ *    mma.sync tensor-core tiles, and one on tcgen05 (TMEM accumulators, the
+ *    query rows as the MMA M dimension, up to 128 rows of a KV head per
+ *    CTA), used when a KV head has more than 32 query rows (and at most 64
+ *    query heads share the KV head).  Sequences are processed
  *    longest context first.
  *    Supported: head_dim in {64, 128}; page_size == 16; rows <= 64;
  *    num_q_heads % num_kv_heads == 0; (num_q_heads / num_kv_heads) * rows <= 512.
@@ -165,8 +166,8 @@ COSPEC_API int cospec_verify_attn_plan(const cospec_attn_dims* dims, int max_ctx
  * `splits` CTAs of one attention kernel variant a device keeps resident at
  * once (0: such a cluster cannot be scheduled).  kernel 0 (mma.sync):
  * `rows` = padded query rows of a CTA (16, 32 or 64), `block_rows` = the
- * block's keys padded to 16; kernel 1 (tcgen05): `rows` = the score tile's
- * query columns (32 or 64), `block_rows` as for kernel 0. */
+ * block's keys padded to 16; kernel 1 (tcgen05): `rows` = 128 (the query
+ * rows of a CTA), `block_rows` as for kernel 0. */
 typedef long long (*cospec_resident_fn)(int kernel, int rows, int block_rows, int splits,
                                         void* user);
 

@@ -17,7 +17,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libcospec.so")
-SOURCES = ["api.cu", "verify_attn.cu", "verify_attn_tc.cu", "lmhead.cu", "arbitrate.cu", "rl.cu",
+SOURCES = ["api.cu", "verify_attn.cu", "verify_attn_tcq.cu", "lmhead.cu", "arbitrate.cu", "rl.cu",
            "accept_commit.cu", "sps.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "--expt-relaxed-constexpr",

@@ -197,18 +197,17 @@ static int check_attn_dims(const cospec_attn_dims* d) {
 // memory, not on the grid).
 static long long resident_clusters(int D, const AttnPlan& pl, int S, int Hkv, int B, int R) {
   // [dev][D==128][variant][block keys / 16 - 1][S - 1]: count + 1 (0: not yet queried)
-  static std::atomic<int> cache[MAX_DEV][2][6][4][16];
+  static std::atomic<int> cache[MAX_DEV][2][5][4][16];
   const int kbr = (R + 15) & ~15;
   int dev = 0;
   cudaGetDevice(&dev);
   const int di = D == 128 ? 1 : 0;
-  const int mi = pl.kind == 1 ? (pl.nt == 32 ? 4 : 5)
-                              : (pl.mt == 1 ? 0 : pl.mt == 2 ? 1 : pl.mt == 4 ? 2 : 3);
+  const int mi = pl.kind == 1 ? 4 : (pl.mt == 1 ? 0 : pl.mt == 2 ? 1 : pl.mt == 4 ? 2 : 3);
   if (S < 1 || S > 16) return 0;
   std::atomic<int>& slot = cache[dev < MAX_DEV ? dev : MAX_DEV - 1][di][mi][kbr / 16 - 1][S - 1];
   int c = slot.load(std::memory_order_relaxed);
   if (c == 0) {
-    c = 1 + (pl.kind == 1 ? attn_tc_max_active_clusters(D, pl.nt, S, Hkv, B, pl.rg)
+    c = 1 + (pl.kind == 1 ? attn_tcq_max_active_clusters(D, S, Hkv, B, pl.rg)
                           : attn_max_active_clusters(D, pl.mt, pl.wk, S, Hkv, B, kbr));
     slot.store(c, std::memory_order_relaxed);
   }
@@ -250,7 +249,7 @@ COSPEC_API int cospec_verify_attn_plan_model(const cospec_attn_dims* d, int max_
       d->batch, d->rows, d->num_q_heads, d->num_kv_heads, d->head_dim, max_ctx, num_sms,
       (d->flags & COSPEC_ATTN_KV_STABLE) != 0,
       [=](const AttnPlan& p, int S) -> long long {
-        return resident(p.kind, p.kind == 1 ? p.nt : p.nrp, kbr, S, user);
+        return resident(p.kind, p.kind >= 1 ? p.nt : p.nrp, kbr, S, user);
       });
   *kernel = pl.kind;
   *splits = pl.cluster;

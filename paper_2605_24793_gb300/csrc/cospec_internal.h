@@ -78,9 +78,9 @@ struct AttnArgs {
   int block_full;  // block rows attend to every block row
 };
 struct AttnPlan {
-  int kind;               // 0: mma.sync kernel, 1: tcgen05 kernel
+  int kind;               // 0: mma.sync kernel, 1: tcgen05 kernel (query rows as MMA M)
   int mt, wk, nrp;        // mma.sync: row tiles, key groups, padded rows
-  int nt, jb, jbq, rg;    // tcgen05: row capacity (32 / 64), block rows per row group,
+  int nt, jb, jbq, rg;    // tcgen05: row capacity (128), block rows per row group,
                           // block rows of the query box, row groups
   int cluster;            // CTAs per (sequence, KV head, row group): the KV split
   long long units;        // (sequence, KV head, row group) units, one cluster each
@@ -95,10 +95,10 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
 int attn_max_active_clusters(int D, int mt, int wk, int S, int Hkv, int B, int kbr);
 cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& plan, int* err,
                                cudaStream_t stream);
-bool tc_attn_supported(int D, int G);
-int attn_tc_max_active_clusters(int D, int nt, int S, int Hkv, int B, int RG);
-cudaError_t launch_verify_attn_tc(const AttnArgs& a, const AttnPlan& plan, int* err,
-                                  cudaStream_t stream);
+bool tcq_attn_supported(int D, int G);
+int attn_tcq_max_active_clusters(int D, int S, int Hkv, int B, int RG);
+cudaError_t launch_verify_attn_tcq(const AttnArgs& a, const AttnPlan& plan, int* err,
+                                   cudaStream_t stream);
 
 // ---------------------------------------------------------------- LM head
 struct LmheadPlan {

@@ -683,28 +683,29 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
   pl.wk = (pl.mt >= 4) ? 1 : 4 / pl.mt;
   pl.nrp = pl.mt * 16;
   const int G = Hq / Hkv;
-  const int jb = G <= 64 ? 64 / G : 1;
-  const int jbq = R < jb ? R : jb;
-  // More than 32 query rows per group: the mma.sync kernel is bound by its
+  // More than 32 query rows per KV head: the mma.sync kernel is bound by its
   // legacy tensor-core rate there and the tcgen05 kernel (one CTA per SM,
-  // deep ring) takes over at every batch size (measured at batch 1, K = 15
-  // and 25, and batch 16, K = 11 and 15, on the Qwen3-8B shape).  Up to 32
-  // rows the mma.sync kernel keeps the latency-bound small batches.
+  // deep ring, every row of a head in one CTA) takes over at every batch
+  // size.  Up to 32 rows the mma.sync kernel keeps the latency-bound small
+  // batches and the two-CTAs-per-SM streaming of the large ones.
   int S = 1;
-  if (tc_attn_supported(D, G) && G * jbq > 32) {
-    // tcgen05 kernel: row groups of whole block rows, at most 64 query rows
+  const int jb = G <= 128 ? 128 / G : 1;
+  const int jbq = R < jb ? R : jb;
+  if (tcq_attn_supported(D, G) && G <= 64 && G * jbq > 32) {
+    // tcgen05 kernel with the query rows as the MMA M dimension: row groups
+    // of whole block rows, at most 128 query rows, so a KV head's rows share
+    // one cache stream (K <= 31 at G = 4, K <= 15 at G = 8)
     pl.kind = 1;
     pl.jb = jb;
     pl.jbq = jbq;
     pl.rg = (R + pl.jb - 1) / pl.jb;
-    pl.nt = ((G * pl.jbq + 15) / 16 * 16) <= 32 ? 32 : 64;
-    // 128-key tiles; one CTA per SM (a stage ring of 96-192 KB); about one
-    // wave of CTAs or a little more (with the longest contexts started first
-    // the tail balances itself and every further split only adds merges:
-    // Qwen3-32B batch 32 ran 238 us unsplit against 255 with 2 splits,
-    // Qwen3-8B batch 16 K = 15 65 us with 2 against 87 with 4), at least
-    // eight tiles per CTA unless the batch is small (the prologue, the query
-    // load and the merge are fixed costs), no CTA with more than 256 tiles.
+    pl.nt = 128;
+    // 128-key tiles; one CTA per SM (a 192 KB stage ring); about one wave
+    // of CTAs or a little more (with the longest contexts started first the
+    // tail balances itself and every further split only adds merges), at
+    // least eight tiles per CTA unless the batch is small (the prologue, the
+    // query load and the merge are fixed costs), no CTA with more than 256
+    // tiles.
     const int tiles_tc = (max_ctx + 127) / 128;
     pl.units = (long long)B * Hkv * pl.rg;
     const long long wave_tc = ((long long)num_sms + pl.units - 1) / (pl.units > 0 ? pl.units : 1);
@@ -714,10 +715,6 @@ AttnPlan plan_verify_attn(int B, int R, int Hq, int Hkv, int D, int max_ctx, int
     // down to two tiles per CTA
     pl.one_wave = (pl.units * 4 <= num_sms && len_tc <= 1) ? 1 : 0;
     if (pl.one_wave) {
-      // the largest split of any size up to 16 whose clusters are all resident
-      // at once (batch 1, K = 15: 12 splits 11.6 us per layer against 12.5 with 8
-      // and 19.7 with 16, a second wave; K = 25, two row groups: 16.5 us with 4
-      // splits, 23.7 with 8, whose 16 clusters do not fit at once)
       int s = 16;
       while (s > 1 && (s * 2 > tiles_tc || resident(pl, s) < pl.units)) --s;
       pl.cluster = s;
@@ -775,7 +772,7 @@ int attn_max_active_clusters(int D, int mt, int wk, int S, int Hkv, int B, int k
 
 cudaError_t launch_verify_attn(const AttnArgs& a, const AttnPlan& pl, int* err,
                                cudaStream_t stream) {
-  if (pl.kind == 1) return launch_verify_attn_tc(a, pl, err, stream);
+  if (pl.kind == 1) return launch_verify_attn_tcq(a, pl, err, stream);
   // Pool as {64 columns, rows, half}: a {64, 16, H} box is one page of one
   // head, both 128-byte halves, landing as [half][16 rows][128 B].
   CUtensorMap maps[4];

@@ -107,8 +107,9 @@ def _gb300_resident(kernel, rows, block_rows, splits):
 # against 2 and 8; Llama-3-8B batch 64: 2 against 4 and 8; Qwen3-32B batch
 # 32: unsplit against 2; Qwen3-8B batch 16 K = 15: 2 against 4; batch 1, K = 5:
 # 16 back to back, 12 alone; batch 2: 12 against 13, 8 and 16; batch 4: 8
-# against 12 and 16; batch 1, K = 15: 12 against 8 and 16; K = 25: 6 against
-# 4 and 8).
+# against 12 and 16; batch 1, K = 15 and K = 25 (one 64- or 104-row group per
+# KV head on the tcgen05 kernel): 12, the largest split whose clusters are
+# all resident at one CTA per SM).
 PLAN_CASES = [
     ((1, 6, 32, 8, 128, 4096, 1), (C.ATTN_MMA_SYNC, 16)),   # Qwen3-8B, batch 1, K = 5
     ((1, 6, 32, 8, 128, 4096, 0), (C.ATTN_MMA_SYNC, 12)),   # the same, on an idle GPU
@@ -116,7 +117,7 @@ PLAN_CASES = [
     ((4, 6, 32, 8, 128, 4096, 1), (C.ATTN_MMA_SYNC, 8)),    # batch 4: 32 clusters at once
     ((16, 8, 32, 8, 128, 8192, 1), (C.ATTN_MMA_SYNC, 4)),   # Qwen3-8B, batch 16, K = 7
     ((1, 16, 32, 8, 128, 4096, 1), (C.ATTN_TCGEN05, 12)),   # batch 1, K = 15: one wave
-    ((1, 26, 32, 8, 128, 4096, 1), (C.ATTN_TCGEN05, 6)),    # batch 1, K = 25: 16 clusters
+    ((1, 26, 32, 8, 128, 4096, 1), (C.ATTN_TCGEN05, 12)),   # batch 1, K = 25: 104 rows, one group
     ((16, 16, 32, 8, 128, 8192, 1), (C.ATTN_TCGEN05, 2)),   # batch 16, K = 15
     ((32, 8, 64, 8, 128, 16384, 1), (C.ATTN_TCGEN05, 1)),   # Qwen3-32B, batch 32
     ((64, 8, 32, 8, 128, 32768, 1), (C.ATTN_MMA_SYNC, 2)),  # Llama-3-8B, batch 64
@@ -146,7 +147,7 @@ def test_attention_plan_model_rules(lib):
     # short contexts: at least four 64-key tiles per CTA (256 keys -> 1 split)
     assert C.verify_attn_plan_model(dims, 256, 152, _gb300_resident) == (0, 1)
     assert C.verify_attn_plan_model(dims, 512, 152, _gb300_resident) == (0, 2)
-    # more than 32 query rows per row group with G <= 64: the tcgen05 kernel;
+    # more than 32 query rows per KV head with G <= 64: the tcgen05 kernel;
     # a KV head shared by 128 query heads stays on the mma.sync kernel
     big = C.AttnDims(4, 8, 64, 8, 128, 16, 300, 1 << 20, 0.0, 0)
     assert C.verify_attn_plan_model(big, 4096, 152, _gb300_resident)[0] == C.ATTN_TCGEN05

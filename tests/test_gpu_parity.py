@@ -59,23 +59,24 @@ ATTN_CASES = [
     (4, 8, 64, 8, 128, [0, 17, 1000, 3333], True),  # G*R = 64 rows, empty and ragged contexts
     (1, 5, 8, 2, 64, [256], False),                 # head_dim 64
     (3, 3, 4, 4, 128, [5, 64, 65], True),           # G = 1, R = 3 -> 3 rows (one 16-row tile)
-    (2, 16, 64, 8, 128, [100, 2000], True),         # G*R = 128 rows (8 warps)
+    (2, 16, 64, 8, 128, [100, 2000], True),         # G*R = 128 rows: one full row group
     (2, 8, 128, 8, 64, [31, 700], False),           # G = 16 -> 128 rows at head_dim 64
     (2, 1, 32, 8, 128, [0, 1], False),              # K = 0: one row per sequence
     (5, 4, 32, 8, 128, [8191, 40, 63, 64, 2049], True),
-    (1, 26, 32, 8, 128, [4096], False),             # K = 25 (the paper's default): 104 rows, 2 groups
-    (2, 32, 128, 8, 64, [300, 1500], True),         # 512 rows per KV head: 8 row groups
+    (1, 26, 32, 8, 128, [4096], False),             # K = 25 (the paper's default): 104 rows, one group
+    (2, 32, 128, 8, 64, [300, 1500], True),         # 512 rows per KV head: 4 row groups of 128
     (2, 2, 128, 1, 128, [500, 1200], True),         # G = 128 (one KV head): 256 rows, mma.sync
 ]
 
 
 def expected_kernel(R, Hq, Hkv, D):
-    """More than 32 query rows per row group (G <= 64, head_dim 64 or 128):
-    the tcgen05 kernel; otherwise the mma.sync kernel."""
+    """More than 32 query rows per KV head (G <= 64, head_dim 64 or 128):
+    the tcgen05 kernel (row groups of up to 128 rows); otherwise the
+    mma.sync kernel."""
     G = Hq // Hkv
     if G > 64 or D not in (64, 128):
         return C.ATTN_MMA_SYNC
-    jb = 64 // G
+    jb = 128 // G
     return C.ATTN_TCGEN05 if G * min(R, jb) > 32 else C.ATTN_MMA_SYNC
 
 # Batches with a (sequence, KV head, row group) per SM and more than 32 query
@@ -84,11 +85,15 @@ _ctx = lambda n, seed: list(np.random.default_rng(seed).integers(0, 700, n))
 ATTN_TC_CASES = [
     (24, 8, 64, 8, 128, [0, 1, 63, 64, 65, 127, 128, 129] + _ctx(16, 1), True),  # G = 8: 64 rows
     (20, 4, 128, 8, 64, _ctx(20, 2), True),         # head_dim 64, G = 16: 64 rows
-    (10, 8, 128, 8, 128, _ctx(10, 3), True),        # 128 rows: two row groups
+    (10, 8, 128, 8, 128, _ctx(10, 3), True),        # 128 rows: one full row group
     (20, 8, 40, 8, 128, _ctx(20, 4), False),        # G = 5: 40 rows
     (20, 16, 32, 8, 128, [2000] + _ctx(19, 5), True),  # G = 4, 16 block rows: 64 rows, longer context
-    (3, 64, 8, 8, 128, [0, 100, 1500], True),        # R = 64, the largest block: 64 rows per group
-    (2, 64, 16, 8, 64, [50, 700], True),             # R = 64, G = 2: two 64-row groups, head_dim 64
+    (3, 64, 8, 8, 128, [0, 100, 1500], True),        # R = 64, the largest block: 64 rows
+    (2, 64, 16, 8, 64, [50, 700], True),             # R = 64, G = 2: 128 rows, head_dim 64
+    (16, 26, 32, 8, 128, _ctx(16, 11), True),        # K = 25 at batch 16: 104 rows, one group
+    (2, 32, 32, 8, 128, [600, 129], True),           # K = 31: exactly 128 rows
+    (2, 33, 32, 8, 128, [300, 50], True),            # 132 rows: groups of 32 and 1 block rows
+    (1, 16, 32, 8, 64, [2000], False),               # head_dim 64 at batch 1: a split of 8
 ]
 
 
@@ -165,11 +170,11 @@ def test_verify_attention_tcgen05_split_matches_oracle(case):
 ATTN_FULL_CASES = [
     # B, R, Hq, Hkv, D, contexts, shuffled, expected kernel
     (1, 17, 32, 8, 128, [4096], False, 1),          # K = 7 region on a Qwen3-4B-like arbitrator
-    (3, 53, 32, 8, 128, [0, 300, 2500], True, 1),   # K = 25 region: 53 rows, 4 block-key groups of 16
+    (3, 53, 32, 8, 128, [0, 300, 2500], True, 1),   # K = 25 region: 212 rows in groups of 128 and 84
     (2, 4, 128, 1, 128, [700, 90], True, 0),        # G = 128: 512 rows in 64-row groups, mma.sync
     (2, 9, 16, 8, 64, [100, 33], True, 0),          # head_dim 64, K = 3 region
     (20, 53, 8, 8, 128, _ctx(20, 6), True, 1),      # G = 1, 53 rows per group: tcgen05 kernel
-    (24, 17, 32, 8, 128, _ctx(24, 7), True, 1),     # G = 4, 64-row groups: tcgen05 kernel
+    (24, 17, 32, 8, 128, _ctx(24, 7), True, 1),     # G = 4, 68 rows in one group: tcgen05 kernel
     (2, 64, 8, 8, 128, [300, 0], True, 1),          # a 64-row region, the largest block
 ]
 
