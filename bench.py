@@ -472,7 +472,7 @@ def measure(cfg, args, env, inp=None, with_cpu=True, with_e2e=True):
     seg = attn_ms + lm_ms + tail_ms
     kern = {
         "verify_attn": {"ms_per_launch": attn_launch_ms, "launches_per_step": cfg.layers,
-                        "kernel": "tcgen05" if attn_kernel == C.ATTN_TCGEN05 else "mma.sync",
+                        "kernel": C.ATTN_KERNEL_NAMES[attn_kernel],
                         "splits": attn_splits,
                         "bytes_per_launch": a_bytes,
                         "gbs": a_bytes / (attn_launch_ms * 1e-3) / 1e9,

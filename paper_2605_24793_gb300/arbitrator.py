@@ -73,7 +73,7 @@ def time_region_attention(cfg: W.RoundConfig, steps: int = 50, warmup: int = 5) 
     return {"workload": cfg.name, "region_rows": cfg.rows, "batch": cfg.batch,
             "context": int(ctx.max()), "layers": cfg.layers, "us_per_layer": us,
             "gbs": (kv_bytes + blk_bytes) / (us * 1e-6) / 1e9,
-            "kernel": "tcgen05" if kernel == C.ATTN_TCGEN05 else "mma.sync", "splits": splits,
+            "kernel": C.ATTN_KERNEL_NAMES[kernel], "splits": splits,
             "device_error": C.get_device_error()}
 
 

@@ -216,6 +216,7 @@ def num_sms() -> int:
 
 
 ATTN_MMA_SYNC, ATTN_TCGEN05 = 0, 1
+ATTN_KERNEL_NAMES = {ATTN_MMA_SYNC: "mma.sync", ATTN_TCGEN05: "tcgen05"}
 
 
 def verify_attn_plan(q, k_pages, page_table, max_ctx: int, kv_stable: bool = False):
