@@ -79,8 +79,9 @@ struct TcqLayout {
   static constexpr int QH = QM * QROWB;             // one half of the query rows
   static constexpr int QOFF = RING;
   static constexpr int MISC = QOFF + H * QH;
-  // barriers: full[NS], empty[NS], q_full, s_full[2], p_full[2], pv_done[2], mma_done, recv_bar
-  static constexpr int NBAR = 2 * NS + 9;
+  // barriers: full_k[NS], full_v[NS], empty_k[NS], empty_v[NS], q_full, s_full[2], p_full[2],
+  // pv_done[2], mma_done, recv_bar
+  static constexpr int NBAR = 4 * NS + 10;
   static constexpr int HOLDER = MISC + NBAR * 8;    // TMEM base address
   static constexpr int FLAGS = HOLDER + 16;         // abort, tiles issued, sequence slot
   static constexpr int ML1 = FLAGS + 64;            // float [2][QM]: group 1's (m_ref, l)
@@ -165,9 +166,13 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
   // 1024-byte aligned base (TMA 128B swizzle, UMMA descriptors), kept as an
   // offset from the shared array so that accesses stay shared-memory ones.
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + LY::MISC);
-  uint64_t* empty = full + NS;
-  uint64_t* q_full = empty + NS;
+  // A stage's K and V halves fill and free separately: K is dead once its
+  // score product completes, well before P.V frees V, so K refills early.
+  uint64_t* full_k = reinterpret_cast<uint64_t*>(smem + LY::MISC);
+  uint64_t* full_v = full_k + NS;
+  uint64_t* empty_k = full_v + NS;
+  uint64_t* empty_v = empty_k + NS;
+  uint64_t* q_full = empty_v + NS;
   uint64_t* s_full = q_full + 1;      // [2]
   uint64_t* p_full = s_full + 2;      // [2]
   uint64_t* pv_done = p_full + 2;     // [2]
@@ -175,8 +180,8 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
   uint64_t* recv_bar = mma_done + 1;  // partials received from the cluster
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(smem + LY::HOLDER);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + LY::FLAGS);
-  volatile int* n_issued = abort_flag + 1;   // tiles the producer loaded (abort tail)
-  volatile int* seq_slot = abort_flag + 2;
+  volatile int* n_issued = abort_flag + 1;   // [2]: tiles whose K / V loads were issued (abort tail)
+  volatile int* seq_slot = abort_flag + 3;
   uint8_t* qs = smem + LY::QOFF;
 
   const int S = (int)cluster_nctarank();
@@ -191,8 +196,10 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
 
   if (tid == 0) {
     for (int s = 0; s < NS; ++s) {
-      mbar_init(&full[s], Q_PROD);         // one arrival per producer warp
-      mbar_init(&empty[s], 1);
+      mbar_init(&full_k[s], 2);            // the two K producer warps
+      mbar_init(&full_v[s], 1);            // the V producer warp
+      mbar_init(&empty_k[s], 1);
+      mbar_init(&empty_v[s], 1);
     }
     mbar_init(q_full, 1);
     for (int i = 0; i < 2; ++i) {
@@ -205,6 +212,7 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
     mbar_init(recv_bar, 1);
     abort_flag[0] = 0;
     abort_flag[1] = 0;
+    abort_flag[2] = 0;
     fence_barrier_init();
   }
   if (warp == Q_MMA_WARP) {
@@ -242,12 +250,17 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
   if (warp < Q_PROD) {
     // ------------------------------------------------------------ producers
     // A warp's bulk copies are processed one after another, which holds one
-    // warp to about 45 GB/s of 2 KB boxes: three warps split each tile's boxes.
+    // warp to about 45 GB/s of 2 KB boxes: warps 0 and 1 split each tile's K
+    // boxes, warp 2 issues its V boxes (needed later, at P.V).
     const int pw = warp;
-    constexpr int NBOX = 2 * H * QPPT;                  // boxes of a full tile
-    constexpr int BPW = (NBOX + Q_PROD - 1) / Q_PROD;   // boxes per producer warp
-    const int e = pw * BPW + lane;                      // this lane's box
-    const bool mine = lane < BPW && e < NBOX;
+    const int tensor = pw == 2 ? 1 : 0;                 // 0: K, 1: V
+    constexpr int NKB = H * QPPT;                       // boxes of a tensor's tile: page x half
+    const int kb0 = tensor ? 0 : pw * (NKB / 2);        // this warp's first box
+    const int nkb = tensor ? NKB : NKB / 2;             // and its boxes per tile
+    const int e = kb0 + lane;                           // this lane's box
+    const bool mine = lane < nkb;
+    uint64_t* my_full = tensor ? full_v : full_k;
+    uint64_t* my_empty = tensor ? empty_v : empty_k;
     if (pw == 0 && lane == 0) {
       tma_prefetch_desc(&map_kp);
       tma_prefetch_desc(&map_vp);
@@ -267,13 +280,13 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
         pid = (e2 < my_pages) ? __ldg(ptab + e2) : 0;
       }
       const int np = min(QPPT, npages - (t_begin + t) * QPPT);
-      // box e: page e / (2H), tensor (e / H) & 1 (K, V), half e % H
-      const int pg = e / (2 * H);
+      // box e of a tensor: page e / H, half e % H
+      const int pg = e / H;
       int pgid = __shfl_sync(0xffffffffu, pid, (t & 3) * QPPT + (pg & 7));
       if (lane == 0) {
         // this warp's boxes within the tile's np pages
-        const int lo = pw * BPW, hi = min(NBOX, min(lo + BPW, np * 2 * H));
-        mbar_arrive_expect_tx(&full[st], (uint32_t)(max(0, hi - lo) * QPAGE * QROWB));
+        const int hi = min(kb0 + nkb, np * H);
+        mbar_arrive_expect_tx(&my_full[st], (uint32_t)(max(0, hi - kb0) * QPAGE * QROWB));
       }
       __syncwarp();
       if (mine && pg < np) {
@@ -281,9 +294,9 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
           set_err(p.err, ERR_PAGE);
           pgid = 0;
         }
-        const int tensor = (e / H) & 1, h = e % H;
+        const int h = e % H;
         tma_load_3d(smem_u32(sb + tensor * LY::KVB + h * (QKT * QROWB) + pg * (QPAGE * QROWB)),
-                    tensor ? (const void*)&map_vp : (const void*)&map_kp, &full[st], 0,
+                    tensor ? (const void*)&map_vp : (const void*)&map_kp, &my_full[st], 0,
                     (pgid * p.Hkv + kvh) * QPAGE, h, pol);
       }
       __syncwarp();
@@ -291,7 +304,7 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
     auto wait_slot = [&](int t) -> bool {
       if (t < NS) return true;
       const int st = t % NS;
-      const bool w = mbar_wait(&empty[st], (uint32_t)((t / NS) - 1) & 1u, Q_WAIT_NS);
+      const bool w = mbar_wait(&my_empty[st], (uint32_t)((t / NS) - 1) & 1u, Q_WAIT_NS);
       return __all_sync(0xffffffffu, w) && !*abort_flag;
     };
     const int pre = min(n, NS);
@@ -329,14 +342,16 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
       if (wait_slot(t)) {
         const int st = t % NS;
         uint8_t* sb = smem + st * LY::STAGE;
+        // one box per tensor: KBR rows from block row 0 of this head, all
+        // halves, landing as [half][KBR rows][128 B]
         if (pw == 0 && lane == 0) {
-          // one box per tensor: KBR rows from block row 0 of this head, all
-          // halves, landing as [half][KBR rows][128 B]
-          mbar_arrive_expect_tx(&full[st], (uint32_t)(2 * H * KBR * QROWB));
-          tma_load_4d(smem_u32(sb), &map_kb, &full[st], 0, b * p.R, 0, kvh, pol);
-          tma_load_4d(smem_u32(sb + LY::KVB), &map_vb, &full[st], 0, b * p.R, 0, kvh, pol);
-        } else if (lane == 0) {
-          mbar_arrive(&full[st]);
+          mbar_arrive_expect_tx(&full_k[st], (uint32_t)(H * KBR * QROWB));
+          tma_load_4d(smem_u32(sb), &map_kb, &full_k[st], 0, b * p.R, 0, kvh, pol);
+        } else if (pw == 1 && lane == 0) {
+          mbar_arrive(&full_k[st]);
+        } else if (pw == 2 && lane == 0) {
+          mbar_arrive_expect_tx(&full_v[st], (uint32_t)(H * KBR * QROWB));
+          tma_load_4d(smem_u32(sb + LY::KVB), &map_vb, &full_v[st], 0, b * p.R, 0, kvh, pol);
         }
         ++issued;
       } else {
@@ -347,7 +362,7 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
       set_err(p.err, ERR_TIMEOUT);
       *abort_flag = 1;
     }
-    if (pw == 0 && lane == 0) *n_issued = issued;
+    if (pw != 1 && lane == 0) n_issued[tensor] = issued;
   } else if (warp == Q_MMA_WARP) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && T > 0) {
@@ -367,6 +382,7 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
           for (int ks = 0; ks < 4; ++ks)
             umma_bf16(tmem_base + (uint32_t)((t & 1) * QKT), smem_desc_sw128(q0 + h * LY::QH + ks * 32),
                       smem_desc_sw128(kb + h * khalf + ks * 32), idesc_qk, (h | ks) != 0 ? 1u : 0u);
+        umma_commit(&empty_k[st]);         // K of this stage is free once S is done
         umma_commit(&s_full[t & 1]);
       };
       auto issue_pv = [&](int u) {
@@ -382,7 +398,7 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
                            tmem_base + (uint32_t)((u & 1) * QKT + ks * 8),
                            tq_desc_mn_sw128(vb + ks * 2048, vhalf), idesc_pv,
                            (u > 1 || ks > 0) ? 1u : 0u);
-        umma_commit(&empty[st]);
+        umma_commit(&empty_v[st]);
         umma_commit(&pv_done[u & 1]);
       };
       // Issue whichever product is ready, so that a P.V product (which frees
@@ -392,26 +408,30 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
       // order, so S may be issued once that product is.  At most one tile's
       // S runs ahead of the oldest pending P.V, which also keeps every
       // barrier within one phase of the parity tested here.
-      int ts = 0, tp = 0;
+      int ts = 0, tp = 0, idle = 0;
       uint64_t t_last = global_timer_ns();
       while (ok && tp < T) {
         bool did = false;
-        if (tp < ts && mbar_test(&p_full[tp & 1], (uint32_t)(tp >> 1) & 1u)) {
+        if (tp < ts && mbar_test(&p_full[tp & 1], (uint32_t)(tp >> 1) & 1u) &&
+            mbar_test(&full_v[tp % NS], (uint32_t)(tp / NS) & 1u)) {
           tc_fence_after();
           issue_pv(tp);
           ++tp;
           did = true;
         }
-        if (ts < T && ts <= tp + 1 && mbar_test(&full[ts % NS], (uint32_t)(ts / NS) & 1u)) {
+        if (ts < T && ts <= tp + 1 && mbar_test(&full_k[ts % NS], (uint32_t)(ts / NS) & 1u)) {
           tc_fence_after();
           issue_s(ts);
           ++ts;
           did = true;
         }
+        // the clock is read only every 256 idle polls (the limit stays bounded)
         if (did) {
-          t_last = global_timer_ns();
-        } else if (*abort_flag || global_timer_ns() - t_last > Q_WAIT_NS) {
-          ok = false;
+          idle = 0;
+        } else if ((++idle & 255) == 0) {
+          const uint64_t now = global_timer_ns();
+          if (idle == 256) t_last = now;
+          else if (*abort_flag || now - t_last > Q_WAIT_NS) ok = false;
         }
       }
       if (!ok) {
@@ -468,8 +488,10 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
         tc_fence_after();
         const uint32_t srow = lane_base + (uint32_t)(grp * QKT);
         // keys 0..lim of this tile are visible to this row (raw scores; the
-        // scale is positive, so it is applied with the exponent)
-        const int lim = !rvalid ? -1 : blk ? blim : min(QKT, C - (t_begin + t) * QKT) - 1;
+        // scale is positive, so it is applied with the exponent).  Padding
+        // rows (r >= NR) give rows of P and O that nothing reads, so they
+        // decide neither the masking nor a rescale.
+        const int lim = blk ? blim : min(QKT, C - (t_begin + t) * QKT) - 1;
         float x[QKT];
 #pragma unroll
         for (int c = 0; c < QKT / 16; ++c) {
@@ -481,7 +503,7 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
           }
         }
         tq_wait_ld();
-        if (__any_sync(0xffffffffu, lim < QKT - 1)) {
+        if (__any_sync(0xffffffffu, rvalid && lim < QKT - 1)) {
 #pragma unroll
           for (int k = 0; k < QKT; ++k) x[k] = (k <= lim) ? x[k] : -INFINITY;
         }
@@ -491,7 +513,7 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
         const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * sc;
         // move the reference only when a score exceeds it by 2^8 (the first
         // tile always sets it: m_ref starts at -inf)
-        const bool up = mx > mref + Q_LAZY;
+        const bool up = rvalid && mx > mref + Q_LAZY;
         float alpha = 1.f;
         if (up) {
           alpha = (mref == -INFINITY) ? 0.f : exp2_approx(mref - mx);
@@ -539,7 +561,9 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
         // stale bytes: zero them so that their zero weights contribute 0.
         {
           const int vr = blk ? p.R : min(QKT, C - (t_begin + t) * QKT);
-          if (vr < nk) {
+          // (V lands separately from K: wait for it before overwriting rows)
+          if (vr < nk &&
+              __all_sync(0xffffffffu, mbar_wait(&full_v[st], (uint32_t)(t / NS) & 1u, Q_WAIT_NS))) {
             uint8_t* vb = sb + LY::KVB;
             const int vhalf = nk * QROWB;
             for (int e = gtid; e < (nk - vr) * H * 8; e += nsw * 32) {
@@ -725,10 +749,13 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
   // After an abort a copy may still be in flight: wait (bounded) for the
   // last fill of every stage the producer used before shared memory goes.
   if (*abort_flag && tid == 0) {
-    const int ni = *n_issued;
-    for (int st = 0; st < NS && st < ni; ++st) {
-      const int last = st + ((ni - 1 - st) / NS) * NS;
-      mbar_wait(&full[st], (uint32_t)(last / NS) & 1u, Q_WAIT_NS);
+    for (int tn = 0; tn < 2; ++tn) {
+      const int ni = n_issued[tn];
+      uint64_t* f = tn ? full_v : full_k;
+      for (int st = 0; st < NS && st < ni; ++st) {
+        const int last = st + ((ni - 1 - st) / NS) * NS;
+        mbar_wait(&f[st], (uint32_t)(last / NS) & 1u, Q_WAIT_NS);
+      }
     }
     if (T > 0) mbar_wait(q_full, 0, Q_WAIT_NS);
   }
