@@ -131,17 +131,56 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------ drafts
-def gpu_drafts(cfg, inp) -> np.ndarray:
+def gpu_drafts(cfg, inp, with_top1: bool = False):
     """Draft ids for the benchmark, synthesised from the target's own top-8
-    (fp32 logits of the bf16 operands, computed once before timing)."""
+    (fp32 logits of the bf16 operands, computed once before timing).  With
+    ``with_top1`` also each row's fp32 top-1 id and its margin to the top-2
+    logit, for the round's self-check."""
     h = inp["hidden"].float()
-    ranked = []
+    ranked, margin = [], []
     for r0 in range(0, h.shape[0], 64):
         logits = h[r0:r0 + 64] @ inp["w"].float().T
-        ranked.append(torch.topk(logits, 8, dim=1).indices.cpu())
-        del logits
+        top = torch.topk(logits, 8, dim=1)
+        ranked.append(top.indices.cpu())
+        margin.append((top.values[:, 0] - top.values[:, 1]).cpu())
+        del logits, top
     ranked = torch.cat(ranked).numpy().reshape(cfg.batch, cfg.rows, 8)
-    return W.synth_drafts(cfg, ranked)
+    draft = W.synth_drafts(cfg, ranked)
+    if with_top1:
+        return draft, ranked[..., 0].reshape(-1), torch.cat(margin).numpy()
+    return draft
+
+
+def self_check(cfg, rnd, top1, margin) -> dict:
+    """The warm-up round checked on the host against what fixes it without
+    the oracle: the LM head's argmax against the fp32 GEMM's top-1 (rows whose
+    fp32 top-1/top-2 margin is below 1e-3 are near ties and may differ), and
+    the accepted lengths and emitted tokens against the prefix rule (Eq. 15)
+    applied to the round's own drafts, argmax and accept decisions: s is the
+    first draft position whose token differs from the target's and was not
+    accepted (K + 1 if none), the emitted tokens are the drafts before it and
+    then the target's token at it."""
+    am = rnd.argmax.cpu().numpy()
+    draft = rnd.draft.cpu().numpy()
+    acc = rnd.accept.cpu().numpy()
+    s_gpu = rnd.accept_len.cpu().numpy()
+    em = rnd.emitted.cpu().numpy()
+    B, K, R = cfg.batch, cfg.k, cfg.rows
+    amr = am.reshape(B, R)
+    tie = margin < 1e-3
+    diff = am != top1
+    follows = True
+    for b in range(B):
+        sb = K + 1
+        for i in range(1, K + 1):
+            if draft[b, i - 1] != amr[b, i - 1] and acc[b, i - 1] == 0:
+                sb = i
+                break
+        want = list(draft[b, :sb - 1]) + [amr[b, sb - 1]] + [-1] * (R - sb)
+        follows &= int(s_gpu[b]) == sb and em[b].tolist() == [int(v) for v in want]
+    return {"argmax_rows": int(am.size), "argmax_equal_fp32_top1": int((~diff).sum()),
+            "argmax_differ_outside_near_ties": int((diff & ~tie).sum()),
+            "near_ties": int(tie.sum()), "accepted_len_and_tokens_follow_eq15": bool(follows)}
 
 
 # ------------------------------------------------------------------ CPU oracle sample
@@ -333,7 +372,7 @@ def measure(cfg, args, env, inp=None, with_cpu=True, with_e2e=True):
         sps_q = torch.from_numpy(q).cuda()
         del q
     else:
-        draft = gpu_drafts(cfg, inp)
+        draft, top1, margin = gpu_drafts(cfg, inp, with_top1=True)
     rnd = VerifyRound(inp, draft, cfg.lam, temperature=args.temperature,
                       seed=W.sample_seed(cfg), sps_q=sps_q)
     rnd.pack_step_io()                    # one host->device and one device->host copy per step
@@ -361,6 +400,8 @@ def measure(cfg, args, env, inp=None, with_cpu=True, with_e2e=True):
     with torch.cuda.stream(stream):
         rnd.run()                                     # eager warm-up, settles kernel attributes
     torch.cuda.synchronize()
+    check = (self_check(cfg, rnd, top1, margin)
+             if not args.sps and args.temperature is None else None)
     g_attn = cap(lambda: ([rnd.restore_context()] + [rnd.attention(l) for l in range(cfg.layers)]))
     g_lm = cap(rnd.lmhead)
 
@@ -573,6 +614,7 @@ def measure(cfg, args, env, inp=None, with_cpu=True, with_e2e=True):
         "roofline": roof, "kernels": kernels_round(kern), "cpu_baseline": cpu, "e2e": e2e,
         "clocks": clk, "gpu_launches": K * rnd.launches_per_round,
         "accepted_len_mean": s_mean,
+        "self_check": check,
         "emitted_tokens_per_s": world * cfg.batch * s_mean / (ms_per_step * 1e-3),
         "accepted_len_of": ("the one synthetic round every step replays (same drafts, "
                             "context restored); python bench.py --sweep and python -m "
