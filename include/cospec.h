@@ -120,8 +120,9 @@ COSPEC_API int cospec_num_sms(void);
  *    mma.sync tensor-core tiles, and one on tcgen05 (TMEM accumulators, the
  *    query rows as the MMA M dimension, up to 128 rows of a KV head per
  *    CTA), used when a KV head has more than 32 query rows (and at most 64
- *    query heads share the KV head).  Sequences are processed
- *    longest context first.
+ *    query heads share the KV head).  Batches of up to 64 sequences are
+ *    processed longest context first; larger ones in index order (a caller
+ *    can order them).
  *    Supported: head_dim in {64, 128}; page_size == 16; rows <= 64;
  *    num_q_heads % num_kv_heads == 0; (num_q_heads / num_kv_heads) * rows <= 512.
  * ------------------------------------------------------------------------ */

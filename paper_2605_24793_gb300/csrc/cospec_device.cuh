@@ -282,6 +282,11 @@ CS_DEV void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
+// Batches up to this size are taken longest context first (the ranking below
+// reads every context length once per candidate pass, O(B^2 / 32) per CTA);
+// larger batches, enough units for many waves, are taken in index order.
+constexpr int RANK_MAX_B = 64;
+
 // The sequence whose context is the `z`-th longest (ties to the lower index):
 // warp 0 ranks every sequence against all others and publishes the answer
 // through `slot` (any shared word nobody writes yet); every thread of the

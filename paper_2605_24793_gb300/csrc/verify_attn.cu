@@ -246,7 +246,7 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 64,
   // Sequences are taken longest context first (blockIdx.z = rank, ties by
   // index), so that the long ones start early and the short ones fill in
   // behind them at the end of the launch.
-  const int b = p.B > 1 ? sequence_by_rank(p.ctx_len, p.B, (int)blockIdx.z, seq_slot)
+  const int b = (p.B > 1 && p.B <= RANK_MAX_B) ? sequence_by_rank(p.ctx_len, p.B, (int)blockIdx.z, seq_slot)
                         : (int)blockIdx.z;
   const int C = p.ctx_len[b];
   const bool bad = (C < 0) || (C > p.max_pages * PAGE);
@@ -587,7 +587,7 @@ __global__ void __launch_bounds__(MT >= 4 && GEN < 2 ? 192 : MT * WK * 32 + 64,
     }
     const int j = (row_g0 + r) / p.G, g = (row_g0 + r) % p.G;
     // the sequence index is read again here rather than kept through the loop
-    const int bo = p.B > 1 ? *seq_slot : (int)blockIdx.z;
+    const int bo = (p.B > 1 && p.B <= RANK_MAX_B) ? *seq_slot : (int)blockIdx.z;
     __nv_bfloat16* dst = p.out + (((size_t)bo * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D + c;
     uint2 pk;
     pk.x = pack_bf16(acc.x, acc.y);

@@ -231,7 +231,7 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
   // Sequences are taken longest context first (blockIdx.z = rank, ties by
   // index), so that the long ones start early and the short ones fill in
   // behind them at the end of the launch.
-  const int b = p.B > 1 ? sequence_by_rank(p.ctx_len, p.B, (int)blockIdx.z, seq_slot)
+  const int b = (p.B > 1 && p.B <= RANK_MAX_B) ? sequence_by_rank(p.ctx_len, p.B, (int)blockIdx.z, seq_slot)
                         : (int)blockIdx.z;
   const int C = p.ctx_len[b];
   const bool bad = (C < 0) || (C > p.max_pages * QPAGE);

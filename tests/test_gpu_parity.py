@@ -82,6 +82,11 @@ def expected_kernel(R, Hq, Hkv, D):
 # Batches with a (sequence, KV head, row group) per SM and more than 32 query
 # rows per group select the tcgen05 kernel.
 _ctx = lambda n, seed: list(np.random.default_rng(seed).integers(0, 700, n))
+# Batches above 64 sequences are taken in index order, not longest first.
+ATTN_CASES += [
+    (80, 6, 32, 8, 128, _ctx(80, 12), True),        # 24 rows: mma.sync kernel
+    (70, 16, 32, 8, 128, _ctx(70, 13), True),       # 64 rows: tcgen05 kernel
+]
 ATTN_TC_CASES = [
     (24, 8, 64, 8, 128, [0, 1, 63, 64, 65, 127, 128, 129] + _ctx(16, 1), True),  # G = 8: 64 rows
     (20, 4, 128, 8, 64, _ctx(20, 2), True),         # head_dim 64, G = 16: 64 rows

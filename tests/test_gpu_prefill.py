@@ -9,7 +9,7 @@ import torch
 from oracle import cospec_oracle as O
 from paper_2605_24793_gb300 import build as BLD
 from paper_2605_24793_gb300 import cospec as C
-from paper_2605_24793_gb300.prefill import ChunkedPrefill
+from paper_2605_24793_gb300.prefill import BlockPrefill, ChunkedPrefill
 
 from .parity_util import assert_close
 
@@ -26,18 +26,20 @@ def _bf16(rng, shape):
     return torch.from_numpy(rng.standard_normal(shape, dtype=np.float32)).to(torch.bfloat16).cuda()
 
 
+@pytest.mark.parametrize("method", [BlockPrefill, ChunkedPrefill], ids=["block", "chunked"])
 @pytest.mark.parametrize("L,B,T,Hq,Hkv,D,region", [
     (2, 2, 200, 8, 2, 64, 9),        # ragged last chunk (200 = 6 x 32 + 8), K = 3 region
     (1, 1, 33, 32, 8, 128, 17),      # one full chunk and one row, K = 7 region
     (1, 3, 96, 16, 8, 128, 53),      # three full chunks, K = 25 region (53 rows)
+    (1, 1, 1000, 8, 2, 128, 17),     # 32 chunks, the last of 8 rows
 ])
-def test_prefill_then_region_matches_dense_hybrid_attention(L, B, T, Hq, Hkv, D, region):
+def test_prefill_then_region_matches_dense_hybrid_attention(method, L, B, T, Hq, Hkv, D, region):
     rng = np.random.default_rng(T * 7 + region)
     G = Hq // Hkv
     q = _bf16(rng, (L, B, T, Hq, D))
     k = _bf16(rng, (L, B, T, Hkv, D))
     v = _bf16(rng, (L, B, T, Hkv, D))
-    pf = ChunkedPrefill(L, B, T, Hq, Hkv, D, extra_tokens=region)
+    pf = method(L, B, T, Hq, Hkv, D, extra_tokens=region)
     out = pf.run(q, k, v)
     torch.cuda.synchronize()
     assert C.get_device_error() == 0
