@@ -19,14 +19,15 @@
 //                             one of two TMEM score buffers,
 //                O += P V     (M = 128 query rows, N = D, K = keys) with P
 //                             read from TMEM (written over its score
-//                             buffer) and V read MN-major from the V tile;
+//                             buffer; three buffers, so S may run two
+//                             tiles ahead of P.V) and V read MN-major from
+//                             the V tile;
 //   warps 4-11 softmax, two groups of four warps (one per TMEM lane quarter)
-//              taking alternate tiles, each into its own O accumulator: a
-//              thread owns one query row, so the row maximum and the row
-//              sum never leave the thread; it turns its row of S into bf16
-//              P in place and rescales its row of O when its reference
-//              maximum moves.  The two accumulators merge row by row at the
-//              end.
+//              sharing every tile, group g its key columns 64 g .. 64 g + 63:
+//              a thread owns one query row and half of its scores; the two
+//              threads of a row swap their half maxima through shared memory,
+//              turn their scores into bf16 P in place and rescale their half
+//              of the row of O when the row's reference maximum moves.
 // Softmax with a lazy reference maximum per row: scores are taken relative
 // to m_ref, set exactly by the first tile; a later tile moves m_ref (and
 // rescales O and l) only when one of its scores exceeds m_ref by more than
@@ -79,13 +80,14 @@ struct TcqLayout {
   static constexpr int QH = QM * QROWB;             // one half of the query rows
   static constexpr int QOFF = RING;
   static constexpr int MISC = QOFF + H * QH;
-  // barriers: full_k[NS], full_v[NS], empty_k[NS], empty_v[NS], q_full, s_full[2], p_full[2],
-  // pv_done[2], mma_done, recv_bar
-  static constexpr int NBAR = 4 * NS + 10;
+  // barriers: full_k[NS], full_v[NS], empty_k[NS], empty_v[NS], q_full, s_full[NSB],
+  // p_full[NSB], pv_done, mma_done, recv_bar
+  static constexpr int NSB = 3;                     // TMEM score buffers
+  static constexpr int NBAR = 4 * NS + 2 * NSB + 4;
   static constexpr int HOLDER = MISC + NBAR * 8;    // TMEM base address
-  static constexpr int FLAGS = HOLDER + 16;         // abort, tiles issued, sequence slot
-  static constexpr int ML1 = FLAGS + 64;            // float [2][QM]: group 1's (m_ref, l)
-  static constexpr int TOTAL = ML1 + 2 * QM * 4;
+  static constexpr int FLAGS = HOLDER + 16;         // abort, tiles issued [2], sequence slot, row-pair votes [8]
+  static constexpr int XCH = FLAGS + 64;            // float [2][QM]: the groups' row maxima / sums
+  static constexpr int TOTAL = XCH + 2 * QM * 4;
   // partial rows after the last tile, in the idle ring: PART [QM], RECV [QM + 15]
   static constexpr int PD = D + 4;                  // O[D], m, l, pad: conflict-free row stores
   static constexpr int ROWP = PD * 4;
@@ -93,10 +95,10 @@ struct TcqLayout {
   static constexpr int RECV = QM * ROWP;
   static_assert(RECV + (QM + 15) * ROWP <= RING, "partials must fit in the ring");
   static_assert(ROWP % 16 == 0, "bulk copies move whole 16-byte chunks");
-  // TMEM columns: score buffers at 0 and 128, the two groups' O at 256 and 256 + D
+  // TMEM columns: score buffers at 0, 128 and 256, O at 384
   static constexpr uint32_t TCOLS = 512u;
-  static constexpr uint32_t OCOL = 256u;
-  static_assert(OCOL + 2 * D <= TCOLS, "two O accumulators after the score buffers");
+  static constexpr uint32_t OCOL = NSB * QKT;
+  static_assert(OCOL + D <= TCOLS, "the O accumulator after the score buffers");
 };
 
 // 32 lanes x 32 bit, 16 consecutive columns per thread (no wait).
@@ -173,15 +175,16 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
   uint64_t* empty_k = full_v + NS;
   uint64_t* empty_v = empty_k + NS;
   uint64_t* q_full = empty_v + NS;
-  uint64_t* s_full = q_full + 1;      // [2]
-  uint64_t* p_full = s_full + 2;      // [2]
-  uint64_t* pv_done = p_full + 2;     // [2]
-  uint64_t* mma_done = pv_done + 2;
+  uint64_t* s_full = q_full + 1;      // [NSB]
+  uint64_t* p_full = s_full + LY::NSB;  // [NSB]
+  uint64_t* pv_done = p_full + LY::NSB;
+  uint64_t* mma_done = pv_done + 1;
   uint64_t* recv_bar = mma_done + 1;  // partials received from the cluster
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(smem + LY::HOLDER);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + LY::FLAGS);
   volatile int* n_issued = abort_flag + 1;   // [2]: tiles whose K / V loads were issued (abort tail)
   volatile int* seq_slot = abort_flag + 3;
+  volatile int* xvote = abort_flag + 4;      // [2 groups][4 quarters]: this tile's waits succeeded
   uint8_t* qs = smem + LY::QOFF;
 
   const int S = (int)cluster_nctarank();
@@ -202,12 +205,11 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
       mbar_init(&empty_v[s], 1);
     }
     mbar_init(q_full, 1);
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < LY::NSB; ++i) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&p_full[i], (uint32_t)nsw);
+      mbar_init(&p_full[i], (uint32_t)(2 * nsw));   // both softmax groups' warps with rows
     }
-    mbar_init(&pv_done[0], 1);
-    mbar_init(&pv_done[1], 1);
+    mbar_init(pv_done, 1);
     mbar_init(mma_done, 1);
     mbar_init(recv_bar, 1);
     abort_flag[0] = 0;
@@ -245,7 +247,6 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
   const int npages = (C + QPAGE - 1) / QPAGE;
   const int KBR = (p.R + 15) & ~15;                  // block keys padded to 16
   float mref = -INFINITY, l = 0.f;                   // softmax threads: this row's m_ref and sum
-  float a0_ = 1.f, a1_ = 0.f;                        // weights of the two groups' O (group 0)
 
   if (warp < Q_PROD) {
     // ------------------------------------------------------------ producers
@@ -380,10 +381,10 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
         for (int h = 0; h < H; ++h)
 #pragma unroll
           for (int ks = 0; ks < 4; ++ks)
-            umma_bf16(tmem_base + (uint32_t)((t & 1) * QKT), smem_desc_sw128(q0 + h * LY::QH + ks * 32),
+            umma_bf16(tmem_base + (uint32_t)((t % LY::NSB) * QKT), smem_desc_sw128(q0 + h * LY::QH + ks * 32),
                       smem_desc_sw128(kb + h * khalf + ks * 32), idesc_qk, (h | ks) != 0 ? 1u : 0u);
         umma_commit(&empty_k[st]);         // K of this stage is free once S is done
-        umma_commit(&s_full[t & 1]);
+        umma_commit(&s_full[t % LY::NSB]);
       };
       auto issue_pv = [&](int u) {
         const int st = u % NS;
@@ -392,34 +393,33 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
         const int nk = blk ? KBR : QKT;
         const uint32_t vhalf = (uint32_t)(nk * QROWB);
         // P of tile u: 16 keys = 8 TMEM columns per step
-        // tiles alternate between the two softmax groups' O accumulators
         for (int ks = 0; ks < nk / 16; ++ks)
-          umma_bf16_tmem_a(tmem_base + LY::OCOL + (uint32_t)((u & 1) * D),
-                           tmem_base + (uint32_t)((u & 1) * QKT + ks * 8),
+          umma_bf16_tmem_a(tmem_base + LY::OCOL,
+                           tmem_base + (uint32_t)((u % LY::NSB) * QKT + ks * 8),
                            tq_desc_mn_sw128(vb + ks * 2048, vhalf), idesc_pv,
-                           (u > 1 || ks > 0) ? 1u : 0u);
+                           (u > 0 || ks > 0) ? 1u : 0u);
         umma_commit(&empty_v[st]);
-        umma_commit(&pv_done[u & 1]);
+        umma_commit(pv_done);
       };
       // Issue whichever product is ready, so that a P.V product (which frees
       // a ring stage for the producer) never waits behind the next tile's
-      // load.  S of tile ts goes to buffer ts & 1, last read (as P) by the
-      // P.V product of tile ts - 2: tcgen05 MMAs of one thread run in issue
-      // order, so S may be issued once that product is.  At most one tile's
-      // S runs ahead of the oldest pending P.V, which also keeps every
+      // load.  S of tile ts goes to buffer ts % 3, last read (as P) by the
+      // P.V product of tile ts - 3: tcgen05 MMAs of one thread run in issue
+      // order, so S may be issued once that product is.  At most two tiles'
+      // S run ahead of the oldest pending P.V, which also keeps every
       // barrier within one phase of the parity tested here.
       int ts = 0, tp = 0, idle = 0;
       uint64_t t_last = global_timer_ns();
       while (ok && tp < T) {
         bool did = false;
-        if (tp < ts && mbar_test(&p_full[tp & 1], (uint32_t)(tp >> 1) & 1u) &&
+        if (tp < ts && mbar_test(&p_full[tp % LY::NSB], (uint32_t)(tp / LY::NSB) & 1u) &&
             mbar_test(&full_v[tp % NS], (uint32_t)(tp / NS) & 1u)) {
           tc_fence_after();
           issue_pv(tp);
           ++tp;
           did = true;
         }
-        if (ts < T && ts <= tp + 1 && mbar_test(&full_k[ts % NS], (uint32_t)(ts / NS) & 1u)) {
+        if (ts < T && ts <= tp + 2 && mbar_test(&full_k[ts % NS], (uint32_t)(ts / NS) & 1u)) {
           tc_fence_after();
           issue_s(ts);
           ++ts;
@@ -444,14 +444,19 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ softmax
-    // Two groups of four warps take alternate tiles (group g the tiles
-    // t = g mod 2, each into its own O accumulator), so two softmax warps
-    // share every SM sub-partition and hide each other's latencies.
+    // Two groups of four warps (one warp per TMEM lane quarter each) share
+    // every tile: group g takes its key columns 64 g .. 64 g + 63.  A thread
+    // owns one query row; the two threads of a row (same lane, warps q and
+    // q + 4) swap their half-tile maxima through shared memory, so both move
+    // the row's reference maximum together and their P, written over their
+    // own columns of the score buffer, share one O accumulator.
     const int sw = warp - Q_SOFT0;
-    const int grp = sw >> 2;             // tiles t with t % 2 == grp
+    const int grp = sw >> 2;             // key-column half of every tile
     const int q = sw & 3;                // TMEM lane quarter of this warp
     const int r = q * 32 + lane;         // this thread's query row
     const int gtid = q * 32 + lane;      // thread index within the group
+    const int kc0 = grp * (QKT / 2);     // first key column of this half
+    float* xch = reinterpret_cast<float*>(smem + LY::XCH);   // [2][QM]
     if (p.kv_stable) {
       // warm L2 with the group's query rows before the producer's TMA
       for (int e = sw * 32 + lane; e < NR * (D * 2 / 128); e += 256) {
@@ -466,51 +471,63 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
     const int blim = p.block_full ? p.R - 1 : min(jr, p.R - 1);
     const float sc = p.scale_log2;
     const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16);
-    const uint32_t ocol = LY::OCOL + (uint32_t)(grp * D);     // this group's O accumulator
-    const int Tg = (T - grp + 1) / 2;                         // tiles of this group
+    const uint32_t ocol = LY::OCOL + (uint32_t)(grp * (D / 2));   // this group's half of O
+    constexpr int HK = QKT / 2;          // key columns of a half
     if (q < nsw) {
-      for (int i = 0; i < Tg; ++i) {
-        const int t = 2 * i + grp;
+      for (int t = 0; t < T; ++t) {
+        const int sb_i = t % LY::NSB;
         const int st = t % NS;
         uint8_t* sb = smem + st * LY::STAGE;
         const bool blk = do_blk && t == n;
         const int nk = blk ? KBR : QKT;          // score columns of this tile
+        // The two warps of a row pair decide an abort together (from both
+        // votes, read after the first exchange barrier), so neither is left
+        // waiting at a barrier the other no longer reaches.
         const bool okw =
-            __all_sync(0xffffffffu, mbar_wait(&s_full[grp], (uint32_t)i & 1u, Q_WAIT_NS)) &&
+            __all_sync(0xffffffffu, mbar_wait(&s_full[sb_i], (uint32_t)(t / LY::NSB) & 1u, Q_WAIT_NS)) &&
             !*abort_flag;
-        if (!okw) {
-          if (lane == 0) {
-            set_err(p.err, ERR_TIMEOUT);
-            *abort_flag = 1;
-          }
-          break;
-        }
+        if (lane == 0) xvote[grp * 4 + q] = okw ? 1 : 0;
         tc_fence_after();
-        const uint32_t srow = lane_base + (uint32_t)(grp * QKT);
+        const uint32_t srow = lane_base + (uint32_t)(sb_i * QKT);
         // keys 0..lim of this tile are visible to this row (raw scores; the
         // scale is positive, so it is applied with the exponent).  Padding
         // rows (r >= NR) give rows of P and O that nothing reads, so they
         // decide neither the masking nor a rescale.
         const int lim = blk ? blim : min(QKT, C - (t_begin + t) * QKT) - 1;
-        float x[QKT];
+        float x[HK];
 #pragma unroll
-        for (int c = 0; c < QKT / 16; ++c) {
-          if (c * 16 < nk) {
-            tq_ld16(srow + c * 16, &x[c * 16]);
+        for (int c = 0; c < HK / 16; ++c) {
+          if (okw && kc0 + c * 16 < nk) {
+            tq_ld16(srow + kc0 + c * 16, &x[c * 16]);
           } else {
 #pragma unroll
             for (int k = 0; k < 16; ++k) x[c * 16 + k] = -INFINITY;
           }
         }
         tq_wait_ld();
-        if (__any_sync(0xffffffffu, rvalid && lim < QKT - 1)) {
+        if (__any_sync(0xffffffffu, rvalid && lim < kc0 + HK - 1)) {
 #pragma unroll
-          for (int k = 0; k < QKT; ++k) x[k] = (k <= lim) ? x[k] : -INFINITY;
+          for (int k = 0; k < HK; ++k) x[k] = (kc0 + k <= lim) ? x[k] : -INFINITY;
         }
         float m4[4] = {x[0], x[1], x[2], x[3]};
 #pragma unroll
-        for (int k = 4; k < QKT; ++k) m4[k & 3] = fmaxf(m4[k & 3], x[k]);
-        const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * sc;
+        for (int k = 4; k < HK; ++k) m4[k & 3] = fmaxf(m4[k & 3], x[k]);
+        const float mh = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+        // the row's maximum over both halves (both threads have read their
+        // scores by the first barrier, so P may then overwrite them; the
+        // second barrier lets the buffer be rewritten at the next tile)
+        xch[grp * QM + r] = mh;
+        named_bar_sync(1 + q, 64);
+        const float mx = fmaxf(mh, xch[(grp ^ 1) * QM + r]) * sc;
+        const bool ok2 = xvote[q] != 0 && xvote[4 + q] != 0;
+        named_bar_sync(1 + q, 64);
+        if (!ok2) {
+          if (lane == 0) {
+            set_err(p.err, ERR_TIMEOUT);
+            *abort_flag = 1;
+          }
+          break;
+        }
         // move the reference only when a score exceeds it by 2^8 (the first
         // tile always sets it: m_ref starts at -inf)
         const bool up = rvalid && mx > mref + Q_LAZY;
@@ -520,15 +537,15 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
           mref = mx;
           l *= alpha;
         }
-        if (__any_sync(0xffffffffu, up && i > 0)) {
-          // this group's O holds its tiles before t: wait for the last of
-          // them, then scale this row
-          const bool okp = __all_sync(
-              0xffffffffu, mbar_wait(&pv_done[grp], (uint32_t)(i - 1) & 1u, Q_WAIT_NS));
+        if (__any_sync(0xffffffffu, up && t > 0)) {
+          // O holds tiles 0..t-1: wait for the last of them, then scale this
+          // group's half of the row
+          const bool okp =
+              __all_sync(0xffffffffu, mbar_wait(pv_done, (uint32_t)(t - 1) & 1u, Q_WAIT_NS));
           tc_fence_after();
           if (okp) {
 #pragma unroll 1
-            for (int c = 0; c < D / 16; ++c) {
+            for (int c = 0; c < D / 32; ++c) {
               float o[16];
               tq_ld16(lane_base + ocol + c * 16, o);
               tq_wait_ld();
@@ -541,13 +558,13 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
             set_err(p.err, ERR_TIMEOUT);
           }
         }
-        // P = 2^(score * scale - m_ref) in bf16, two keys per TMEM column,
-        // over this row's scores (masked keys give exactly 0)
+        // P = 2^(score * scale - m_ref) in bf16, two keys per TMEM column, in
+        // this half's columns of the score buffer (masked keys give exactly 0)
         const float nb = (mref == -INFINITY) ? 0.f : -mref;
         float l4[4] = {0.f, 0.f, 0.f, 0.f};
-        uint32_t pk[QKT / 2];
+        uint32_t pk[HK / 2];
 #pragma unroll
-        for (int k = 0; k < QKT / 2; ++k) {
+        for (int k = 0; k < HK / 2; ++k) {
           const float p0 = exp2_approx(fmaf(x[2 * k], sc, nb));
           const float p1 = exp2_approx(fmaf(x[2 * k + 1], sc, nb));
           l4[k & 3] += p0 + p1;
@@ -555,13 +572,13 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
         }
         l += (l4[0] + l4[1]) + (l4[2] + l4[3]);
 #pragma unroll
-        for (int c = 0; c < QKT / 32; ++c)
-          if (c * 32 < nk) tq_st16(srow + c * 16, &pk[c * 16]);
+        for (int c = 0; c < HK / 32; ++c)
+          if (kc0 + c * 32 < nk) tq_st16(srow + kc0 / 2 + c * 16, &pk[c * 16]);
         // V rows of keys outside the context (or past the block) may hold
-        // stale bytes: zero them so that their zero weights contribute 0.
-        {
+        // stale bytes: group 0 zeroes them so that their zero weights
+        // contribute 0 (V lands separately from K: wait for it first).
+        if (grp == 0) {
           const int vr = blk ? p.R : min(QKT, C - (t_begin + t) * QKT);
-          // (V lands separately from K: wait for it before overwriting rows)
           if (vr < nk &&
               __all_sync(0xffffffffu, mbar_wait(&full_v[st], (uint32_t)(t / NS) & 1u, Q_WAIT_NS))) {
             uint8_t* vb = sb + LY::KVB;
@@ -577,11 +594,11 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
         tq_wait_st();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&p_full[grp]);
+        if (lane == 0) mbar_arrive(&p_full[sb_i]);
       }
-      if (Tg > 0 && !*abort_flag) {
-        const bool okp = __all_sync(
-            0xffffffffu, mbar_wait(&pv_done[grp], (uint32_t)(Tg - 1) & 1u, Q_WAIT_NS));
+      if (T > 0 && !*abort_flag) {
+        const bool okp =
+            __all_sync(0xffffffffu, mbar_wait(pv_done, (uint32_t)(T - 1) & 1u, Q_WAIT_NS));
         if (!okp && lane == 0) {
           set_err(p.err, ERR_TIMEOUT);
           *abort_flag = 1;
@@ -589,21 +606,12 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
       }
       tc_fence_after();
     }
-    // the second group hands its (m_ref, l) to the first, which merges the
-    // two accumulators row by row below
-    float* ml1 = reinterpret_cast<float*>(smem + LY::ML1);    // [2][QM]
-    if (grp == 1) {
-      ml1[r] = mref;
-      ml1[QM + r] = l;
-    }
-    named_bar_sync(1, 256);
-    if (grp == 0) {
-      const float m1 = ml1[r], l1 = ml1[QM + r];
-      const float M = fmaxf(mref, m1);
-      a0_ = (M == -INFINITY || mref == -INFINITY) ? 0.f : exp2_approx(mref - M);
-      a1_ = (M == -INFINITY || m1 == -INFINITY) ? 0.f : exp2_approx(m1 - M);
-      l = l * a0_ + l1 * a1_;
-      mref = M;
+    // the row's sum over both halves (the exchange buffer is free: every
+    // tile's second barrier has passed)
+    if (q < nsw) {
+      xch[grp * QM + r] = l;
+      named_bar_sync(1 + q, 64);
+      l += xch[(grp ^ 1) * QM + r];
     }
   }
   __syncthreads();
@@ -621,27 +629,16 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
     cluster_arrive_relaxed();
   }
   float* part = reinterpret_cast<float*>(smem + LY::PART);
-  if (warp >= Q_SOFT0 && warp < Q_SOFT0 + 4 && warp - Q_SOFT0 < nsw) {
-    // group 0: O = a0 O_0 + a1 O_1 for this row (the second group's
-    // accumulator holds something only when there were two tiles or more)
-    const int q = warp - Q_SOFT0, r = q * 32 + lane;
+  if (warp >= Q_SOFT0 && ((warp - Q_SOFT0) & 3) < nsw) {
+    // each group writes its half of the row's columns (both hold m_ref and l)
+    const int sw = warp - Q_SOFT0, grp = sw >> 2, q = sw & 3, r = q * 32 + lane;
     const bool rvalid = r < NR;
-    const bool two = T >= 2;
+    const int c0 = grp * (D / 32);       // first 16-column chunk of this group's half
     const uint32_t orow = tmem_base + ((uint32_t)(q * 32) << 16) + LY::OCOL;
     auto load_o = [&](int c, float (&o)[16]) {
       if (have) {
         tq_ld16(orow + c * 16, o);
-        if (two) {
-          float o1[16];
-          tq_ld16(orow + D + c * 16, o1);
-          tq_wait_ld();
-#pragma unroll
-          for (int i = 0; i < 16; ++i) o[i] = o[i] * a0_ + o1[i] * a1_;
-        } else {
-          tq_wait_ld();
-#pragma unroll
-          for (int i = 0; i < 16; ++i) o[i] *= a0_;
-        }
+        tq_wait_ld();
       } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) o[i] = 0.f;
@@ -652,7 +649,7 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
       __nv_bfloat16* dst = p.out + (((size_t)b * p.R + j) * p.Hq + (size_t)kvh * p.G + g) * D;
       const float inv = (have && l > 0.f) ? 1.f / l : 0.f;
 #pragma unroll 1
-      for (int c = 0; c < D / 16; ++c) {
+      for (int c = c0; c < c0 + D / 32; ++c) {
         float o[16];
         load_o(c, o);
         if (rvalid) {
@@ -672,7 +669,7 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
     } else {
       float* prow = part + r * PD;
 #pragma unroll 1
-      for (int c = 0; c < D / 16; ++c) {
+      for (int c = c0; c < c0 + D / 32; ++c) {
         float o[16];
         load_o(c, o);
         if (rvalid) {
@@ -681,7 +678,7 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
             *reinterpret_cast<float4*>(prow + c * 16 + i) = make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]);
         }
       }
-      if (rvalid) {
+      if (rvalid && grp == 0) {
         prow[D] = have ? mref : -INFINITY;
         prow[D + 1] = have ? l : 0.f;
       }
