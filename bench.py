@@ -737,7 +737,7 @@ def main():
 TRAFFIC = {
     ("llama3_8b_b64_k7_mm30", "verify_attn"): 5224876672.0,
     ("qwen3_8b_b1", "verify_attn"): 16920320.0,
-    ("qwen3_32b_b32", "verify_attn"): 1363145472.0,
+    ("qwen3_32b_b32", "verify_attn"): 1362836992.0,
 }
 
 
