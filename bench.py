@@ -735,8 +735,8 @@ def main():
 # full-size launches; Qwen3-32B: one launch of a two-layer run (the
 # per-layer shapes of the full workload).
 TRAFFIC = {
-    ("llama3_8b_b64_k7_mm30", "verify_attn"): 5224876672.0,
-    ("qwen3_8b_b1", "verify_attn"): 16920320.0,
+    ("llama3_8b_b64_k7_mm30", "verify_attn"): 5224868480.0,
+    ("qwen3_8b_b1", "verify_attn"): 16918272.0,
     ("qwen3_32b_b32", "verify_attn"): 1362836992.0,
 }
 
