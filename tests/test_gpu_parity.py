@@ -543,6 +543,77 @@ def test_device_checks_set_error_bits_without_faulting():
     assert C.get_device_error() == 0                       # reading clears the word
 
 
+def test_tcgen05_attention_device_checks_skip_only_the_bad_sequence():
+    # 64 query rows per KV head: the tcgen05 kernel.  A page id outside the
+    # pool (clamped to page 0 for the copy) and a context past the page table
+    # (no tiles at all) each set their bit; the other sequence's rows still
+    # match the oracle.
+    rng = np.random.default_rng(6)
+    t = _paged_case(rng, 2, 16, 32, 8, 128, [700, 300], True)
+    assert C.verify_attn_plan(t["q"], t["k_pages"], t["page_table"], 700)[0] == C.ATTN_TCGEN05
+    ref = O.verify_attention(host(t["q"]), host(t["k_blk"]), host(t["v_blk"]), host(t["k_pages"]),
+                             host(t["v_pages"]), t["table_np"], t["ctx_np"], 16)
+    out = torch.empty_like(t["q"])
+    bad = t["page_table"].clone()
+    bad[1, 5] = 10 ** 6
+    C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], bad, t["ctx_len"],
+                  out, 700)
+    assert C.get_device_error() == C.DEVERR_PAGE
+    assert_close(host(out)[0], ref[0], "attention (tcgen05), the sequence with valid pages")
+    long_ctx = torch.tensor([700, t["table_np"].shape[1] * 16 + 1], dtype=torch.int32, device="cuda")
+    out.fill_(1.0)
+    C.verify_attn(t["q"], t["k_blk"], t["v_blk"], t["k_pages"], t["v_pages"], t["page_table"],
+                  long_ctx, out, 700)
+    assert C.get_device_error() == C.DEVERR_CTX
+    assert_close(host(out)[0], ref[0], "attention (tcgen05), the sequence with a valid context")
+    assert torch.all(out[1] == 0)                          # the skipped sequence attends nothing
+
+
+def test_accept_commit_device_checks_skip_only_the_bad_sequence():
+    # Sequence 1 would run past its page table (ctx + s > capacity): its
+    # context stays, nothing of it is written.  Sequence 2's commit page is
+    # outside the pool: those cells are skipped.  Sequence 0 commits exactly
+    # as the oracle does.
+    rng = np.random.default_rng(41)
+    B, K, L, Hkv, D, P = 3, 3, 2, 8, 128, 16
+    R = K + 1
+    pages_per_seq = 4
+    table = rng.permutation(B * pages_per_seq).astype(np.int32).reshape(B, pages_per_seq)
+    ctx = np.array([37, pages_per_seq * P - 2, 21], dtype=np.int32)
+    table_bad = table.copy()
+    table_bad[2, ctx[2] // P] = 10 ** 6
+    V = 50
+    am = rng.integers(0, V, (B, R)).astype(np.int32)
+    draft = am[:, :K].copy()                               # every draft matches: s = K + 1
+    acc = np.ones((B, K), dtype=np.uint8)
+    num = B * pages_per_seq
+    kb = bf16(rng.standard_normal((L, B, R, Hkv, D)))
+    vb = bf16(rng.standard_normal((L, B, R, Hkv, D)))
+    kp = bf16(rng.standard_normal((L, num, Hkv, P, D)))
+    vp = bf16(rng.standard_normal((L, num, Hkv, P, D)))
+    bits = lambda x: x.cpu().view(torch.int16).numpy()
+    kp0, vp0 = bits(kp), bits(vp)
+    ctx_t = torch.from_numpy(ctx).cuda()
+    alen = torch.empty(B, dtype=torch.int32, device="cuda")
+    em = torch.empty((B, R), dtype=torch.int32, device="cuda")
+    C.accept_commit(torch.from_numpy(draft).cuda(), torch.from_numpy(am).cuda(),
+                    torch.from_numpy(acc).cuda(), kb, vb, kp, vp, torch.from_numpy(table_bad).cuda(),
+                    ctx_t, alen, em)
+    assert C.get_device_error() == C.DEVERR_CTX | C.DEVERR_PAGE
+    s, emitted = O.accept_scan(draft, am, acc)
+    assert np.array_equal(alen.cpu().numpy(), s) and np.array_equal(em.cpu().numpy(), emitted)
+    got_ctx = ctx_t.cpu().numpy()
+    assert got_ctx[0] == ctx[0] + R and got_ctx[1] == ctx[1]
+    # the oracle commit of sequence 0 alone
+    only0 = np.array([R, 0, 0], dtype=np.int64)
+    kp_ref, vp_ref, _ = O.commit_kv(bits(kb), bits(vb), kp0, vp0, table, ctx, only0, P)
+    kp_got, vp_got = bits(kp), bits(vp)
+    for b in range(B):                                     # sequence 2 wrote nothing either
+        pages = table[b]
+        assert np.array_equal(kp_got[:, pages], kp_ref[:, pages])
+        assert np.array_equal(vp_got[:, pages], vp_ref[:, pages])
+
+
 # ---------------------------------------------------------------------------
 # Stochastic decoding: temperature sampling in the LM-head epilogue (Sec. 3.1)
 # ---------------------------------------------------------------------------

@@ -95,6 +95,37 @@ def test_sps_accept_matches_oracle(B, K, V, T, noise):
     assert np.array_equal(target.cpu().numpy().reshape(B, R)[ok], ref["target"][ok])
 
 
+def test_sps_accept_rejects_a_draft_id_outside_the_vocabulary():
+    # The acceptance kernel checks the draft ids itself: an id outside
+    # [0, V) sets the token bit, reads no q or p for it, and is rejected;
+    # the other sequences decide as the oracle does.
+    B, K, V, T = 6, 4, 2000, 1.0
+    cfg, hidden, w, x, q, draft, seed = _sps_case(B, K, V, T, 1.0)
+    R = K + 1
+    ref = S.sps_round(x, q.astype(np.float64), draft, seed, T)
+    dfr = torch.from_numpy(W.draft_for_rows(draft)).cuda()    # the LM head sees valid ids
+    _, st, logits = _lmhead_logits(hidden, w, dfr, T)
+    bad = draft.copy()
+    bad[2, 0] = V + 5
+    target = torch.full((B * R,), -7, dtype=torch.int32, device="cuda")
+    accept = torch.full((B, K), 7, dtype=torch.uint8, device="cuda")
+    ratio = torch.empty((B, K), dtype=torch.float32, device="cuda")
+    seed_t = torch.tensor([seed], dtype=torch.int64, device="cuda")
+    C.sps_accept(torch.from_numpy(bad).cuda(), st, logits, torch.from_numpy(q).cuda(), seed_t,
+                 target, accept, ratio, C.new_sps_workspace(B))
+    torch.cuda.synchronize()
+    assert C.get_device_error() == C.DEVERR_TOKEN
+    acc = accept.cpu().numpy()
+    assert acc[2, 0] == 0
+    tgt = target.cpu().numpy().reshape(B, R)
+    assert np.all((tgt[2] >= -1) & (tgt[2] < V))
+    ties = ((ref["margin"] < TIE) | (ref["key_margin"] < TIE)).astype(np.int64)
+    ok = ties == 0
+    ok[2] = False
+    assert np.array_equal(acc[ok], ref["accept"][ok])
+    assert np.array_equal(tgt[ok], ref["target"][ok])
+
+
 def test_sps_round_with_commit_matches_oracle():
     """A whole round: attention, LM head with logits, speculative-sampling
     acceptance, accept/commit, against the oracle's round and commit."""
