@@ -67,3 +67,16 @@ def test_reference_arm_under_torchrun_prints_once():
     assert r.returncode == 0, r.stderr[-2000:]
     lines = _json_lines(r.stdout)
     assert len(lines) == 1 and lines[0]["impl"] == "reference" and lines[0]["n_gpus"] == 2
+
+
+def test_throttled_clock_records_are_taken_again():
+    # the rule bench.py applies to its own clock record before it prints
+    sys.path.insert(0, ROOT)
+    import bench
+    ok = {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": []}
+    assert not bench.throttled(ok)
+    assert not bench.throttled({"sm_mhz": 1900.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"]})
+    for r in ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"):
+        assert bench.throttled({"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": [r]})
+    assert bench.throttled({"sm_mhz": 1200.0, "sm_max_mhz": 2070.0, "reasons": []})   # a clock lock
+    assert not bench.throttled({"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]})
