@@ -16,7 +16,7 @@
 //              own K/V as a final tile;
 //   warp 3     MMA issuer (one thread):
 //                S  = Q K^T   (M = 128 query rows, N = 128 keys, K = D) into
-//                             one of two TMEM score buffers,
+//                             one of three TMEM score buffers,
 //                O += P V     (M = 128 query rows, N = D, K = keys) with P
 //                             read from TMEM (written over its score
 //                             buffer; three buffers, so S may run two
