@@ -86,6 +86,8 @@ _ctx = lambda n, seed: list(np.random.default_rng(seed).integers(0, 700, n))
 ATTN_CASES += [
     (80, 6, 32, 8, 128, _ctx(80, 12), True),        # 24 rows: mma.sync kernel
     (70, 16, 32, 8, 128, _ctx(70, 13), True),       # 64 rows: tcgen05 kernel
+    (64, 4, 32, 8, 128, _ctx(64, 15), True),        # 64 sequences: the largest batch ranked
+    (65, 4, 32, 8, 128, _ctx(65, 16), True),        # 65: the smallest taken in index order
 ]
 ATTN_TC_CASES = [
     (24, 8, 64, 8, 128, [0, 1, 63, 64, 65, 127, 128, 129] + _ctx(16, 1), True),  # G = 8: 64 rows
@@ -99,6 +101,9 @@ ATTN_TC_CASES = [
     (2, 32, 32, 8, 128, [600, 129], True),           # K = 31: exactly 128 rows
     (2, 33, 32, 8, 128, [300, 50], True),            # 132 rows: groups of 32 and 1 block rows
     (1, 16, 32, 8, 64, [2000], False),               # head_dim 64 at batch 1: a split of 8
+    (2, 3, 64, 1, 128, [400, 1000], True),           # G = 64, the largest: row groups of 2 and 1 block rows
+    (3, 11, 24, 8, 128, [129, 700, 0], True),        # G = 3: 33 rows, one past the mma.sync kernel
+    (64, 8, 64, 8, 128, _ctx(64, 14), True),         # 64 sequences, ranked longest first
 ]
 
 
