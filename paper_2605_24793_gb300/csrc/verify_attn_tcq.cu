@@ -12,9 +12,9 @@
 // by warp:
 //   warps 0-2  TMA producers: 128-key K/V tiles (one 2-D box per page and
 //              128-byte half: [half][128 keys][128 B], 128B-swizzled) into a
-//              3-stage ring, the query rows of the group once, the block's
-//              own K/V as a final tile;
-//   warp 3     MMA issuer (one thread):
+//              3-stage ring, the block's own K/V as a final tile;
+//   warp 3     MMA issuer (one thread), which first loads the query rows of
+//              the group:
 //                S  = Q K^T   (M = 128 query rows, N = 128 keys, K = D) into
 //                             one of three TMEM score buffers,
 //                O += P V     (M = 128 query rows, N = D, K = keys) with P
@@ -322,14 +322,9 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
           tma_prefetch_l2_3d((lane & 1) ? (const void*)&map_vp : (const void*)&map_kp, 0,
                              (pg * p.Hkv + kvh) * QPAGE, h);
     }
-    // the query rows and the block K/V come from the previous kernel; the
-    // other producers read only the (stable) cache
+    // the block K/V comes from the previous kernel; the other producers
+    // read only the (stable) cache
     if (p.kv_stable && pw == 0) griddep_wait();
-    if (T > 0 && pw == 0 && lane == 0) {
-      mbar_arrive_expect_tx(q_full, (uint32_t)(H * qrows * QROWB));
-      for (int h = 0; h < H; ++h)
-        tma_load_4d(smem_u32(qs + h * LY::QH), &map_q, q_full, 0, kvh * p.G, b * p.R + j0, h, pol);
-    }
     for (int t = pre; t < n && ok; ++t) {
       if (!wait_slot(t)) {
         ok = false;
@@ -369,6 +364,18 @@ __global__ void __launch_bounds__(Q_THREADS, 1)
     if (lane == 0 && T > 0) {
       const uint32_t idesc_pv = idesc_bf16_f32(QM, D) | (1u << 16);   // B (V) MN-major
       const uint32_t q0 = smem_u32(qs);
+      {
+        // The query rows come from the previous kernel: this thread loads
+        // them as soon as that kernel is done, while the producer warps are
+        // still issuing the first cache tiles (a warp's bulk copies run one
+        // after another; behind three tiles' boxes the rows landed ~2 us
+        // later at batch 1).
+        if (p.kv_stable) griddep_wait();
+        const uint64_t qpol = p.RG > 1 ? l2_policy_evict_normal() : l2_policy_evict_first();
+        mbar_arrive_expect_tx(q_full, (uint32_t)(H * qrows * QROWB));
+        for (int h = 0; h < H; ++h)
+          tma_load_4d(smem_u32(qs + h * LY::QH), &map_q, q_full, 0, kvh * p.G, b * p.R + j0, h, qpol);
+      }
       bool ok = mbar_wait(q_full, 0, Q_WAIT_NS);
       auto issue_s = [&](int t) {
         const int st = t % NS;
