@@ -760,7 +760,7 @@ def main():
 TRAFFIC = {
     ("llama3_8b_b64_k7_mm30", "verify_attn"): 5224868480.0,
     ("qwen3_8b_b1", "verify_attn"): 16918272.0,
-    ("qwen3_32b_b32", "verify_attn"): 1362836992.0,
+    ("qwen3_32b_b32", "verify_attn"): 1362597120.0,
 }
 
 
