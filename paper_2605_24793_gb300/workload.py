@@ -330,3 +330,48 @@ def sample_from(cfg: RoundConfig, q: np.ndarray, round_index: int = 0) -> np.nda
     cdf = np.cumsum(q, axis=-1)
     r = rng.random(q.shape[:-1] + (1,)) * cdf[..., -1:]
     return np.minimum(np.sum(cdf < r, axis=-1), q.shape[-1] - 1).astype(np.int32)
+
+
+# ------------------------------------------------------------------ replay
+_BF16_KEYS = ("q", "k_blk", "v_blk", "k_pages", "v_pages", "hidden", "w")
+
+
+def save_inputs(path: str, inp: Dict[str, object], draft: Optional[np.ndarray] = None) -> None:
+    """Write one round's inputs (and optionally its draft ids) to ``path``
+    as an uncompressed ``.npz``, bf16 tensors as their 16-bit patterns, so
+    that a case (a failing parity shape, say) can be replayed bit for bit
+    without its generator.  Nothing is computed; there is no model state to
+    checkpoint, since every input of a round is one of these arrays."""
+    import json
+    arrays = {k: inp[k].detach().cpu().contiguous().view(torch.int16).numpy()
+              for k in _BF16_KEYS}
+    w1, b1, w2, b2 = inp["mlp"]
+    arrays.update(mlp_w1=w1.cpu().numpy(), mlp_b1=b1.cpu().numpy(), mlp_w2=w2.cpu().numpy(),
+                  mlp_b2=np.asarray(float(b2), dtype=np.float32),
+                  ctx_len_np=np.asarray(inp["ctx_len_np"]), page_table_np=np.asarray(inp["page_table_np"]),
+                  num_pages=np.asarray(int(inp["num_pages"])),
+                  alias_layers=np.asarray(bool(inp.get("alias_layers", False))),
+                  cfg_json=np.asarray(json.dumps(dataclasses.asdict(inp["cfg"]))))
+    if draft is not None:
+        arrays["draft"] = np.asarray(draft, dtype=np.int32)
+    np.savez(path, **arrays)
+
+
+def load_inputs(path: str, device="cpu"):
+    """Read what ``save_inputs`` wrote: (inputs as ``make_round_inputs``
+    returns them, on ``device``; the draft ids or None)."""
+    import json
+    device = torch.device(device)
+    with np.load(path, allow_pickle=False) as z:
+        out: Dict[str, object] = dict(
+            cfg=RoundConfig(**json.loads(str(z["cfg_json"]))),
+            ctx_len_np=z["ctx_len_np"].copy(), page_table_np=z["page_table_np"].copy(),
+            num_pages=int(z["num_pages"]), alias_layers=bool(z["alias_layers"]))
+        for k in _BF16_KEYS:
+            out[k] = torch.from_numpy(z[k].copy()).view(torch.bfloat16).to(device)
+        out["mlp"] = (torch.from_numpy(z["mlp_w1"].copy()), torch.from_numpy(z["mlp_b1"].copy()),
+                      torch.from_numpy(z["mlp_w2"].copy()), torch.tensor(float(z["mlp_b2"])))
+        out["page_table"] = torch.from_numpy(out["page_table_np"]).to(device)
+        out["ctx_len"] = torch.from_numpy(out["ctx_len_np"]).to(device)
+        draft = z["draft"].copy() if "draft" in z.files else None
+    return out, draft

@@ -130,3 +130,28 @@ def test_rl_batch_records():
     assert ro[0] == 0 and np.all(np.diff(ro) >= 1) and np.all(np.diff(ro) <= 6)
     assert m.shape == a.shape == ell.shape == (ro[-1], 7)
     assert np.all(a[m == 1] == 1) and np.all(ell <= 0)
+
+
+def test_saved_inputs_replay_bit_for_bit(tmp_path):
+    # a round's inputs and drafts written to .npz and read back are the same
+    # bits, and the oracle's round on them gives the same result
+    from oracle import cospec_oracle as O
+    cfg = W.CONFIGS["tiny"].replace(batch=2, k=3, ctx_lo=20, ctx_hi=70, shuffled_pages=True)
+    inp = W.make_round_inputs(cfg)
+    x = O.lmhead_logits(inp["hidden"], inp["w"])
+    draft = W.synth_drafts(cfg, O.topk_ids(x, 8).reshape(cfg.batch, cfg.rows, 8))
+    path = str(tmp_path / "round.npz")
+    W.save_inputs(path, inp, draft)
+    got, got_draft = W.load_inputs(path)
+    assert got["cfg"] == cfg and got["num_pages"] == inp["num_pages"]
+    assert np.array_equal(got_draft, draft)
+    assert np.array_equal(got["ctx_len_np"], inp["ctx_len_np"])
+    assert np.array_equal(got["page_table_np"], inp["page_table_np"])
+    for k in ("q", "k_blk", "v_blk", "k_pages", "v_pages", "hidden", "w"):
+        assert got[k].dtype == torch.bfloat16 and torch.equal(got[k].view(torch.int16), inp[k].view(torch.int16))
+    for a, b in zip(got["mlp"], inp["mlp"]):
+        assert torch.equal(a, b)
+    ref = O.cospec_round(inp, draft, 0.6)
+    rep = O.cospec_round(got, got_draft, 0.6)
+    for k in ("s", "emitted", "p"):
+        assert np.array_equal(np.asarray(rep[k]), np.asarray(ref[k]), equal_nan=True), k
