@@ -195,6 +195,29 @@ def self_check(cfg, rnd, top1, margin) -> dict:
             "near_ties": int(tie.sum()), "accepted_len_and_tokens_follow_eq15": bool(follows)}
 
 
+def mismatch_stats(cfg, rnd) -> dict:
+    """How the round's arbitration treated the draft/target mismatches
+    (Sec. 3.3): positions i in 1..K whose draft token differs from the
+    target's prediction, how many of them the policy accepted (a_i = 1),
+    and how many of those accepted ones lie before the round's first
+    rejection, i.e. reached the emitted block."""
+    if cfg.k == 0:
+        return {"mismatch_positions": 0, "mismatches_accepted": 0, "accepted_mismatch_fraction": None,
+                "accepted_mismatches_emitted": 0}
+    R = cfg.rows
+    am = rnd.argmax.cpu().numpy().reshape(cfg.batch, R)[:, :cfg.k]
+    draft = rnd.draft.cpu().numpy()
+    acc = rnd.accept.cpu().numpy().astype(bool)
+    s = rnd.accept_len.cpu().numpy()
+    mism = draft != am
+    kept = mism & acc
+    before = np.arange(1, cfg.k + 1)[None, :] < s[:, None]      # positions i < s_b
+    n = int(mism.sum())
+    return {"mismatch_positions": n, "mismatches_accepted": int(kept.sum()),
+            "accepted_mismatch_fraction": (float(kept.sum()) / n) if n else None,
+            "accepted_mismatches_emitted": int((kept & before).sum())}
+
+
 # ------------------------------------------------------------------ CPU oracle sample
 class OracleSampler:
     """Times the CPU oracle on a bounded, seeded sample of one round.
@@ -414,6 +437,7 @@ def measure(cfg, args, env, inp=None, with_cpu=True, with_e2e=True):
     torch.cuda.synchronize()
     check = (self_check(cfg, rnd, top1, margin)
              if not args.sps and args.temperature is None else None)
+    mism = mismatch_stats(cfg, rnd) if not args.sps else None
     g_attn = cap(lambda: ([rnd.restore_context()] + [rnd.attention(l) for l in range(cfg.layers)]))
     g_lm = cap(rnd.lmhead)
 
@@ -638,6 +662,7 @@ def measure(cfg, args, env, inp=None, with_cpu=True, with_e2e=True):
         "clocks": clk, "gpu_launches": K * rnd.launches_per_round,
         "accepted_len_mean": s_mean,
         "self_check": check,
+        "mismatches": mism,
         "emitted_tokens_per_s": world * cfg.batch * s_mean / (ms_per_step * 1e-3),
         "accepted_len_of": ("the one synthetic round every step replays (same drafts, "
                             "context restored); python bench.py --sweep and python -m "
@@ -680,6 +705,7 @@ def run_sweep(args, env):
                 "workload": cfg.name, "k": cfg.k, "mismatch_rate": cfg.mismatch_rate,
                 "batch": cfg.batch, "layers": cfg.layers,
                 "tau": res["tau"], "rounds": res["rounds"],
+                "mismatches_first_round": line.get("mismatches"),
                 "decode_ms_per_round": res["ms_per_round"],
                 "decode_emitted_tokens_per_s": res["emitted_tokens_per_s"],
                 "block_tokens_per_s": line["value"], "ms_per_step": line["ms_per_step"],

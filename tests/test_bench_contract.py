@@ -80,3 +80,24 @@ def test_throttled_clock_records_are_taken_again():
         assert bench.throttled({"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": [r]})
     assert bench.throttled({"sm_mhz": 1200.0, "sm_max_mhz": 2070.0, "reasons": []})   # a clock lock
     assert not bench.throttled({"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]})
+
+
+def test_mismatch_stats_counts_what_the_arbitration_kept():
+    # a hand-built round: K = 3, two sequences
+    #   seq 0: drafts [5, 7, 9] vs targets [5, 8, 1]: mismatches at 2 and 3,
+    #          position 2 accepted, 3 rejected -> s = 3; one kept, before s
+    #   seq 1: drafts [1, 2, 3] vs targets [4, 2, 6]: mismatches at 1 and 3,
+    #          both accepted -> s = 4; two kept, both before s
+    import types
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2605_24793_gb300 import workload as W
+    cfg = W.CONFIGS["tiny"].replace(batch=2, k=3)
+    rnd = types.SimpleNamespace(
+        argmax=torch.tensor([5, 8, 1, 0, 4, 2, 6, 0], dtype=torch.int32),
+        draft=torch.tensor([[5, 7, 9], [1, 2, 3]], dtype=torch.int32),
+        accept=torch.tensor([[1, 1, 0], [1, 1, 1]], dtype=torch.uint8),
+        accept_len=torch.tensor([3, 4], dtype=torch.int32))
+    st = bench.mismatch_stats(cfg, rnd)
+    assert st == {"mismatch_positions": 4, "mismatches_accepted": 3,
+                  "accepted_mismatch_fraction": 0.75, "accepted_mismatches_emitted": 3}
